@@ -1,0 +1,404 @@
+"""Benchmark of the one-GPU doubly pipelined, dual-root reduction-to-all.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+                    [--kernel fused|schedule] [--b B] [--impl reference]
+
+A step is one reduction-to-all of p rank vectors of m elements: every rank's
+y_i receives x_0 (.) ... (.) x_{p-1} (one launch of the fused kernel, or of
+the schedule kernel with --kernel schedule).  Inputs are seeded synthetic
+vectors generated on the device before timing (counter-based generator of
+paper_2109_12626_gb300.inputs).  The metric is GB/s = 2 p m sizeof / t (p m
+elements read plus p m written) over K timed steps after W warm-up steps;
+the inputs (and outputs) are larger than the 129 MB L2, so no flush is
+needed between steps.
+
+The JSON line also carries
+  e2e           the same metric with pinned host buffers: per step the host
+                to device copy of all p inputs, the kernel, and the device
+                to host copy of all p outputs (dpdr_allreduce_host);
+  roofline      achieved HBM bytes per launch / launch time (CUDA events on
+                the launch stream) against the measured copy bandwidth;
+  cpu_baseline  the CPU oracle (tree fold + copy to p rows, one thread) on a
+                bounded column sample of the same workload;
+  clocks        nvidia-smi samples taken during the timed region.
+
+--impl reference times the CPU oracle itself on the host cores (the
+reference arm; rank 0 only under torchrun).  Under torchrun with N > 1 every
+rank runs an independent replica of the workload on its own GPU (the path
+has no cross-GPU exchange); time is the max over ranks and value the total
+over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+DEFAULT_WORKLOAD = "p32_m134217728_f32"
+METRIC = "allreduce GB/s (p*m*sizeof read + p*m*sizeof written)"
+ESIZE = {"int32": 4, "float32": 4, "mat2x2u32": 16}
+DTYPE_TAG = {"int32": "int32", "float32": "f32", "mat2x2u32": "u32"}
+KERNEL_SOURCES = {"fused": "fused.cu", "schedule": "schedule.cu"}
+
+
+# ------------------------------------------------------------ workload
+def workload(name: str, m_override: int | None = None) -> dict:
+    from paper_2109_12626_gb300.inputs import WORKLOADS
+    w = dict(WORKLOADS[name])
+    if m_override:
+        w["m"] = int(m_override)
+    if w["m"] is None:
+        w["m"] = 1 << 23
+    return w
+
+
+def gen_device_inputs(w, dev):
+    import torch
+    from paper_2109_12626_gb300 import inputs as I
+    kw = I.workload_kwargs(w)
+    xs = []
+    for i in range(w["p"]):
+        v = I.rank_values(w["kind"], w["seed"], i, w["m"], device=dev, **kw)
+        xs.append(v.reshape(-1).contiguous())
+        del v
+    torch.cuda.synchronize()
+    return xs
+
+
+# --------------------------------------------------------- distributed
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    """Largest value over all ranks (the slowest rank's time)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int) -> None:
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# -------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int, period_ms: int = 100):
+        self.proc = None
+        self.gpu = gpu_index
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(gpu_index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", str(period_ms)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self) -> dict | None:
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=10)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        return summarize_clocks(out)
+
+
+def summarize_clocks(csv_text: str) -> dict | None:
+    rows = []
+    for line in csv_text.strip().splitlines():
+        f = [x.strip() for x in line.split(",")]
+        if len(f) < 9:
+            continue
+        try:
+            rows.append(dict(sm=float(f[1]), max=float(f[2]),
+                             power=float(f[3]) if f[3] not in ("[N/A]", "N/A") else 0.0,
+                             hw=f[5], hwt=f[6], swt=f[7], cap=f[8]))
+        except ValueError:
+            continue
+    if not rows:
+        return None
+    load = [r for r in rows if r["power"] > 200.0] or rows
+    reasons = set()
+    for r in load:
+        for k, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                        ("swt", "sw_thermal_slowdown"), ("cap", "sw_power_cap")):
+            if r[k].lower() == "active":
+                reasons.add(name)
+    return {"sm_mhz": statistics.median(r["sm"] for r in load),
+            "sm_max_mhz": max(r["max"] for r in load),
+            "reasons": sorted(reasons), "samples": len(load)}
+
+
+# ------------------------------------------------------------ roofline
+def measured_peak_gbs() -> tuple[float, str]:
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+def kernel_source_hash(kernel: str) -> str:
+    h = hashlib.sha256()
+    for f in (KERNEL_SOURCES[kernel], "ops.cuh"):
+        with open(os.path.join(ROOT, "paper_2109_12626_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel: str, wname: str, units: int) -> float | None:
+    """DRAM bytes per launch from the committed ncu summary, scaled to the
+    units of this launch; None if the kernel changed since the capture."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)[kernel][wname]
+    except (OSError, KeyError, ValueError):
+        return None
+    if rec.get("source_hash") != kernel_source_hash(kernel):
+        return None
+    return float(rec["bytes_per_unit"]) * units
+
+
+# --------------------------------------------------------- CPU oracle
+def cpu_sample(w: dict, target_s: float = 12.0, max_cols: int | None = None):
+    """Time the oracle (tree fold + copy to all p rows) single-threaded on a
+    column sample of the workload; returns (GB/s, description, reps)."""
+    import numpy as np
+    import torch
+    from oracle import oracle as O
+    from paper_2109_12626_gb300 import inputs as I
+    p, kind = w["p"], w["kind"]
+    es = ESIZE[kind]
+    cols = max(1, min(w["m"], (1 << 24) // p if max_cols is None else max_cols))
+    kw = I.workload_kwargs(w)
+    x = torch.stack([I.rank_values(kind, w["seed"], i, cols, **kw) for i in range(p)])
+    x = x.numpy()
+    dt = {"int32": O.I32, "float32": O.F32, "mat2x2u32": O.MAT}[kind]
+    if kind == "mat2x2u32":
+        x = x.view(np.uint32).reshape(p, cols, 4)
+    y = np.empty_like(x)
+    O.allreduce(x, dt, out=y)  # warm
+    reps, t0 = 0, time.perf_counter()
+    while True:
+        O.allreduce(x, dt, out=y)
+        reps += 1
+        el = time.perf_counter() - t0
+        if el >= target_s or reps >= 1000:
+            break
+    gbs = 2.0 * p * cols * es * reps / el / 1e9
+    return gbs, "%d ranks x %d of %d columns, %d repetitions" % (p, cols, w["m"], reps), el / reps
+
+
+def run_reference(args, w) -> dict:
+    """The reference arm: the CPU oracle on the host cores, K timed steps of
+    a bounded sample of the workload after W warm-up steps."""
+    import numpy as np
+    import torch
+    from oracle import oracle as O
+    from paper_2109_12626_gb300 import inputs as I
+    p, kind = w["p"], w["kind"]
+    es = ESIZE[kind]
+    cols = max(1, min(w["m"], (1 << 22) // p))
+    kw = I.workload_kwargs(w)
+    x = torch.stack([I.rank_values(kind, w["seed"], i, cols, **kw) for i in range(p)]).numpy()
+    dt = {"int32": O.I32, "float32": O.F32, "mat2x2u32": O.MAT}[kind]
+    if kind == "mat2x2u32":
+        x = x.view(np.uint32).reshape(p, cols, 4)
+    y = np.empty_like(x)
+    for _ in range(args.warmup):
+        O.allreduce(x, dt, out=y)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        O.allreduce(x, dt, out=y)
+    el = time.perf_counter() - t0
+    v = 2.0 * p * cols * es * args.steps / el / 1e9
+    sample = "%d ranks x %d of %d columns per step" % (p, cols, w["m"])
+    return {"impl": "reference", "metric": METRIC, "value": round(v, 4), "unit": "GB/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(el / args.steps * 1e3, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": DTYPE_TAG[kind],
+            "data": "synthetic (seeded counter-based generator)",
+            "config": {"workload": args.workload, "p": p, "m": w["m"], "sample_columns": cols},
+            "cpu_baseline": {"value": round(v, 4), "unit": "GB/s", "cores": 1,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(v, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+# ---------------------------------------------------------------- main
+def main(argv=None) -> int:
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--m", type=int, default=None, help="override m (sweeps)")
+    ap.add_argument("--kernel", choices=("fused", "schedule"), default="fused")
+    ap.add_argument("--b", type=int, default=None, help="pipeline blocks (schedule)")
+    ap.add_argument("--mode", type=int, default=0, help="fused layout: 0 auto, 1, 2")
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    args = ap.parse_args(argv)
+    args.warmup = max(args.warmup, 3)
+
+    world, rank, local = dist_env()
+    w = workload(args.workload, args.m)
+
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args, w)), flush=True)
+        return 0
+
+    import torch
+    import paper_2109_12626_gb300 as pkg
+    from paper_2109_12626_gb300 import build as B
+
+    assert torch.cuda.is_available(), "bench.py needs a GPU"
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    if not os.path.exists(B.LIB):
+        B.build()
+
+    p, m, kind = w["p"], w["m"], w["kind"]
+    es = ESIZE[kind]
+    b = args.b if args.b is not None else (w.get("b") or 0)
+    xs = gen_device_inputs(w, dev)
+    ys = [torch.empty_like(x) for x in xs]
+    plan = pkg.Plan(p, m, kind, b)
+    if args.mode:
+        plan.set(pkg.OPT_FUSED_MODE, args.mode)
+    stream = torch.cuda.current_stream(dev)
+    run = plan.allreduce if args.kernel == "fused" else plan.allreduce_schedule
+    algo_bytes = 2 * p * m * es
+
+    for _ in range(args.warmup):
+        run(xs, ys, stream)
+    plan.sync(stream)
+
+    sampler = ClockSampler(local)
+    time.sleep(0.3)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    start.record(stream)
+    for k in range(args.steps):
+        ev[k][0].record(stream)
+        run(xs, ys, stream)
+        ev[k][1].record(stream)
+    stop.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clocks = sampler.stop()
+    plan.sync(stream)
+    total_ms = start.elapsed_time(stop)
+    launch_ms = [a.elapsed_time(z) for a, z in ev]
+    t_max = max_over_ranks(total_ms, world, dev)
+    ms_per_step = t_max / args.steps
+    value = world * algo_bytes / (ms_per_step * 1e-3) / 1e9
+    avg_launch = sum(launch_ms) / len(launch_ms)
+    achieved = algo_bytes / (avg_launch * 1e-3) / 1e9
+    peak, peak_kind = measured_peak_gbs()
+    units = p * m
+    traffic = profiled_traffic(args.kernel, args.workload, units)
+
+    # end to end with host buffers
+    e2e = None
+    if not args.no_e2e:
+        xh = [torch.empty(x.shape, dtype=x.dtype, pin_memory=True) for x in xs]
+        yh = [torch.empty(x.shape, dtype=x.dtype, pin_memory=True) for x in xs]
+        for h, x in zip(xh, xs):
+            h.copy_(x)
+        for _ in range(2):
+            plan.allreduce_host(xh, yh, xs, ys, stream)
+        plan.sync(stream)
+        k2 = max(3, min(args.steps, 10))
+        barrier(world)
+        torch.cuda.synchronize(dev)
+        s2, e2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s2.record(stream)
+        for _ in range(k2):
+            plan.allreduce_host(xh, yh, xs, ys, stream)
+        e2.record(stream)
+        torch.cuda.synchronize(dev)
+        t2 = max_over_ranks(s2.elapsed_time(e2), world, dev) / k2
+        e2e = {"value": round(world * algo_bytes / (t2 * 1e-3) / 1e9, 3), "unit": "GB/s",
+               "h2d_bytes_per_step": p * m * es, "d2h_bytes_per_step": p * m * es,
+               "steps": k2, "ms_per_step": round(t2, 3)}
+        del xh, yh
+
+    cpu = None
+    if rank == 0 and not args.no_cpu:
+        gbs, sample, _ = cpu_sample(w, args.cpu_seconds)
+        cpu = {"value": round(gbs, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+               "sample": sample}
+
+    info = plan.info()
+    line = {
+        "metric": METRIC, "value": round(value, 2), "unit": "GB/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": DTYPE_TAG[kind],
+        "data": "synthetic (seeded counter-based generator, generated on device)",
+        "config": {"workload": args.workload, "p": p, "m": m, "kind": kind,
+                   "kernel": args.kernel, "b": info["b"],
+                   "fused_mode": args.mode or info["auto_mode"],
+                   "bytes_per_step": algo_bytes,
+                   "l2": "inputs larger than L2 (%.1f GB), no flush" % (algo_bytes / 2e9)
+                   if algo_bytes / 2 > 129e6 else "working set fits L2: warm-cache number",
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+                     "unit": "GB/s", "frac": round(achieved / peak, 4),
+                     "peak_kind": peak_kind + " copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
+                     "traffic": traffic,
+                     "kernel_ms": round(avg_launch, 4)},
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": args.steps,
+        "clocks": clocks,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    plan.close()
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

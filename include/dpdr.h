@@ -1,0 +1,193 @@
+/*
+ * dpdr.h -- C ABI of a one-GPU doubly pipelined, dual-root reduction-to-all
+ * (J. L. Traff, "A Doubly-pipelined, Dual-root Reduction-to-all Algorithm
+ * and Implementation", arXiv 2109.12626, 2021).
+ *
+ * The operation (Sec. 1, problem statement): each of p successively ranked
+ * processors holds a vector x_i of m elements; the element-wise product
+ * y = x_0 (.) x_1 (.) ... (.) x_{p-1} for an associative, not necessarily
+ * commutative operator (.) is computed and delivered to all p processors.
+ * Here the p processors are virtual ranks on one GPU: rank i is an input
+ * buffer x[i] and an output buffer y[i], each m elements in device memory.
+ *
+ * The result is the bracketing of Sec. 1.1 and Algorithm 1: the ranks form
+ * two post-order-numbered complete binary trees, tree 0 = ranks
+ * [0, floor(p/2)) and tree 1 = [floor(p/2), p); the value of node i is
+ * v(child_1) (.) ( v(child_0) (.) x_i ) with child_0 = i-1, and
+ * y = v(r0) (.) v(r1) for the roots r0 = floor(p/2)-1 and r1 = p-1.  Every
+ * entry point below produces exactly this result, bit for bit, for every
+ * element type (float32 included), in every y[i].
+ *
+ * Conventions for all functions:
+ *   - Status codes (dpdr_status) are returned; nothing throws, the device
+ *     never traps.  A failing call also sets a thread-local last error
+ *     (dpdr_last_error, dpdr_last_error_message).
+ *   - "host array of p device pointers": x and y are arrays in host memory
+ *     holding p device addresses; the caller owns every buffer, each of
+ *     m elements of the plan's element type, contiguous.  Every buffer must
+ *     be aligned to its element size (4 bytes); 16-byte alignment of all
+ *     2p buffers enables the vectorised path.
+ *   - In-place use, y[i] == x[i] (Algorithm 1 initialises Y <- x_i and
+ *     leaves y in Y), is allowed for every i.  Any other overlap between
+ *     buffers is invalid.
+ *   - Calls are asynchronous on the given stream; the inputs must stay
+ *     valid and unmodified until the stream has passed the call.
+ */
+#ifndef DPDR_H
+#define DPDR_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Element types and operators (the operator functors of the library). */
+typedef enum {
+    DPDR_INT32 = 0,      /* int32, sum wraps mod 2^32                       */
+    DPDR_FLOAT32 = 1,    /* IEEE float32, sum rounded to nearest even        */
+    DPDR_MAT2X2_U32 = 2  /* 2x2 uint32 matrix, row-major a,b,c,d (16 bytes) */
+} dpdr_dtype;
+
+typedef enum {
+    DPDR_OP_SUM = 0,     /* with DPDR_INT32 or DPDR_FLOAT32                  */
+    DPDR_OP_MATMUL = 1   /* with DPDR_MAT2X2_U32: product mod 2^32, the lower
+                            rank on the left (non-commutative)              */
+} dpdr_op;
+
+typedef enum {
+    DPDR_OK = 0,
+    DPDR_ERR_INVALID = 1,          /* bad argument, alignment or overlap     */
+    DPDR_ERR_CUDA = 2,             /* a CUDA runtime call failed             */
+    DPDR_ERR_TIMEOUT = 3,          /* a bounded wait of the schedule kernel
+                                      expired (reported by dpdr_plan_sync)   */
+    DPDR_ERR_NOT_COOPERATIVE = 4,  /* the schedule kernel's CTAs cannot all
+                                      be resident at once                    */
+    DPDR_ERR_OOM = 5               /* device or pinned host memory exhausted */
+} dpdr_status;
+
+/* Opaque plan; owns the device-side tables and scratch of one (p, m, type). */
+typedef struct dpdr_plan_s* dpdr_plan_t;
+
+/* A CUDA stream (cudaStream_t / CUstream); NULL is the legacy default
+ * stream. */
+typedef struct CUstream_st* dpdr_stream_t;
+
+/* ---------------------------------------------------------------- host only
+ * These need no GPU. */
+
+/* The dual post-order trees of Sec. 1.1 for p ranks.  Fills five
+ * caller-owned int[p] arrays: parent (-1 at the roots), child0 (= i-1 when
+ * i has a child, else -1), child1 (the root of the lower subtree interval,
+ * -1 if none; a node with one child has only child0), dual (the other root
+ * at r0 and r1, else -1) and depth (d_i, 0 at the roots; Algorithm 1 runs
+ * rounds j = 0..b+d_i).  Any pointer may be NULL.  p >= 1. */
+int dpdr_tree(int p, int* parent, int* child0, int* child1, int* dual,
+              int* depth);
+
+/* Block partition of Algorithm 1 (Sec. 1.1: b successive blocks of roughly
+ * m/b elements): writes b+1 caller-owned starts, block j = [starts[j],
+ * starts[j+1]); the first m mod b blocks hold ceil(m/b) elements, the rest
+ * floor(m/b).  Requires 1 <= b <= m. */
+int dpdr_blocks(int64_t m, int b, int64_t* starts);
+
+/* Block count from the pipelining-lemma optimum of Sec. 1.2,
+ * b* = sqrt((4h-6) m beta / (3 alpha)) with h = ceil(log2(p+2)), written
+ * with kappa = alpha/beta in elements: round(sqrt((4h-6) m / (3 kappa))),
+ * clamped to [1, max(m,1)].  kappa <= 0 selects the default 1024. */
+int dpdr_block_count_rule(int p, int64_t m, double kappa);
+
+/* -------------------------------------------------------------------- plan */
+
+/* Builds the trees, the block partition and the device tables for p ranks
+ * of m elements of (dtype, op) on the current CUDA device, and allocates the
+ * plan's device scratch (rank-pointer tables, handshake counters, the dual
+ * roots' exchange slots, an error word).  b is the number of pipeline
+ * blocks (Algorithm 1); b == 0 selects dpdr_block_count_rule(p, m, 0);
+ * b is clamped to [1, max(m,1)].  p >= 1, m >= 0.  Returns NULL on error
+ * (see dpdr_last_error).  Not thread-safe with respect to one plan. */
+dpdr_plan_t dpdr_plan(int p, int64_t m, dpdr_dtype dtype, dpdr_op op, int b);
+
+/* Copies the plan's trees (caller-owned int[p] arrays, any may be NULL) and
+ * the block count in use. */
+int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
+                    int* dual, int* depth, int* b_used);
+
+/* Plan options (key, value):
+ *   DPDR_OPT_FUSED_MODE       0 auto, 1 column-streaming, 2 shared-memory
+ *                             tile (the two layouts of dpdr_allreduce)
+ *   DPDR_OPT_WAIT_LIMIT_NS    bound of every wait of the schedule kernel,
+ *                             nanoseconds (default 4e9)
+ *   DPDR_OPT_SKIP_RANK        fault injection for tests: this rank of the
+ *                             schedule kernel never publishes a block, so
+ *                             its partners' waits expire (-1 = off)
+ *   DPDR_OPT_SCHED_THREADS    threads per CTA of the schedule kernel
+ *                             (64..256, multiple of 32; default 128)
+ *   DPDR_OPT_SCHED_RANKS_PER_CTA  virtual ranks per CTA (0 = fewest that
+ *                             fit co-resident)
+ *   DPDR_OPT_BLOCKS           change b (same rules as dpdr_plan's b) */
+enum {
+    DPDR_OPT_FUSED_MODE = 1,
+    DPDR_OPT_WAIT_LIMIT_NS = 2,
+    DPDR_OPT_SKIP_RANK = 3,
+    DPDR_OPT_SCHED_THREADS = 4,
+    DPDR_OPT_SCHED_RANKS_PER_CTA = 5,
+    DPDR_OPT_BLOCKS = 6
+};
+int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
+
+/* Plan facts for tools and tests, int64 each, n of them:
+ *   [0] p  [1] m  [2] b  [3] max depth  [4] fused mode that auto selects
+ *   [5] schedule CTAs  [6] ranks per schedule CTA  [7] device scratch bytes
+ *   [8] 1 if the last dpdr_allreduce ran the 16-byte vector path */
+int dpdr_plan_info(dpdr_plan_t plan, int64_t* info, int n);
+
+/* Releases the plan's device and host memory.  The caller must first make
+ * sure no call on the plan is still running on the GPU.  NULL is a no-op. */
+void dpdr_plan_destroy(dpdr_plan_t plan);
+
+/* --------------------------------------------------------------- run it */
+
+/* Fused bandwidth kernel: y[i] = y for all i, one kernel launch.  Each
+ * element column is read once from each of the p inputs and written once to
+ * each of the p outputs (2 p m element transfers of device memory); the
+ * (.)-combines follow the bracketing above exactly.  x, y: host arrays of p
+ * device pointers.  Asynchronous on stream. */
+int dpdr_allreduce(dpdr_plan_t plan, const void* const* x, void* const* y,
+                   dpdr_stream_t stream);
+
+/* Schedule-faithful kernel: runs Algorithm 1 for every virtual rank, rounds
+ * j = 0..b+d_i, each round's exchanges with child_0, child_1 and the parent
+ * or dual, as one cooperative persistent launch in which CTAs own ranks and
+ * exchange pipeline blocks through device memory with release/acquire
+ * counters.  Same result as dpdr_allreduce.  Every wait is bounded
+ * (DPDR_OPT_WAIT_LIMIT_NS); an expired wait ends the kernel early and is
+ * reported as DPDR_ERR_TIMEOUT by dpdr_plan_sync.  Returns
+ * DPDR_ERR_NOT_COOPERATIVE if the ranks cannot be co-resident.
+ * Asynchronous on stream. */
+int dpdr_allreduce_schedule(dpdr_plan_t plan, const void* const* x,
+                            void* const* y, dpdr_stream_t stream);
+
+/* Host buffers end to end: copies x_host[i] (pinned or pageable host
+ * memory) into the device buffers x_dev[i], runs dpdr_allreduce into y_dev,
+ * and copies y_dev[i] back into y_host[i], all on stream.  All four are
+ * host arrays of p pointers. */
+int dpdr_allreduce_host(dpdr_plan_t plan, const void* const* x_host,
+                        void* const* y_host, void* const* x_dev,
+                        void* const* y_dev, dpdr_stream_t stream);
+
+/* Waits for stream, then reports and clears any device-side error of the
+ * plan's schedule kernel: DPDR_ERR_TIMEOUT with details in
+ * dpdr_last_error_message ("rank r round j step s"). */
+int dpdr_plan_sync(dpdr_plan_t plan, dpdr_stream_t stream);
+
+/* ------------------------------------------------------------ errors */
+int dpdr_last_error(void);
+const char* dpdr_last_error_message(void);
+const char* dpdr_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DPDR_H */

@@ -1,0 +1,207 @@
+"""ctypes binding of libdpdr.so (the C ABI of include/dpdr.h).
+
+The library is loaded on first use from this package's directory; it is
+built by ``paper_2109_12626_gb300.build`` (or ``__graft_entry__.build()``).
+There is no fallback: without the library every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Sequence
+
+import numpy as np
+
+DPDR_INT32, DPDR_FLOAT32, DPDR_MAT2X2_U32 = 0, 1, 2
+DPDR_OP_SUM, DPDR_OP_MATMUL = 0, 1
+(DPDR_OK, DPDR_ERR_INVALID, DPDR_ERR_CUDA, DPDR_ERR_TIMEOUT,
+ DPDR_ERR_NOT_COOPERATIVE, DPDR_ERR_OOM) = range(6)
+(OPT_FUSED_MODE, OPT_WAIT_LIMIT_NS, OPT_SKIP_RANK, OPT_SCHED_THREADS,
+ OPT_SCHED_RANKS_PER_CTA, OPT_BLOCKS) = range(1, 7)
+
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libdpdr.so")
+
+# every function the header declares, with its ctypes signature
+_P = ctypes.c_void_p
+_IP = ctypes.POINTER(ctypes.c_int)
+_I64P = ctypes.POINTER(ctypes.c_int64)
+SIGNATURES = {
+    "dpdr_tree": (ctypes.c_int, [ctypes.c_int, _IP, _IP, _IP, _IP, _IP]),
+    "dpdr_blocks": (ctypes.c_int, [ctypes.c_int64, ctypes.c_int, _I64P]),
+    "dpdr_block_count_rule": (ctypes.c_int, [ctypes.c_int, ctypes.c_int64,
+                                             ctypes.c_double]),
+    "dpdr_plan": (_P, [ctypes.c_int, ctypes.c_int64, ctypes.c_int,
+                       ctypes.c_int, ctypes.c_int]),
+    "dpdr_plan_query": (ctypes.c_int, [_P, _IP, _IP, _IP, _IP, _IP, _IP]),
+    "dpdr_plan_set": (ctypes.c_int, [_P, ctypes.c_int, ctypes.c_int64]),
+    "dpdr_plan_info": (ctypes.c_int, [_P, _I64P, ctypes.c_int]),
+    "dpdr_plan_destroy": (None, [_P]),
+    "dpdr_allreduce": (ctypes.c_int, [_P, _P, _P, _P]),
+    "dpdr_allreduce_schedule": (ctypes.c_int, [_P, _P, _P, _P]),
+    "dpdr_allreduce_host": (ctypes.c_int, [_P, _P, _P, _P, _P, _P]),
+    "dpdr_plan_sync": (ctypes.c_int, [_P, _P]),
+    "dpdr_last_error": (ctypes.c_int, []),
+    "dpdr_last_error_message": (ctypes.c_char_p, []),
+    "dpdr_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+}
+
+_lib = None
+
+
+class DpdrError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        msg = lib().dpdr_last_error_message().decode(errors="replace")
+        name = lib().dpdr_status_string(status).decode()
+        super().__init__("%s: %s (%d): %s" % (where, name, status, msg))
+
+
+def lib():
+    """The loaded library (raises if it was not built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(
+                "libdpdr.so is not built; run `python -m "
+                "paper_2109_12626_gb300.build` (no CPU fallback exists)")
+        L = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in SIGNATURES.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _check(rc: int, where: str) -> None:
+    if rc != DPDR_OK:
+        raise DpdrError(rc, where)
+
+
+def tree(p: int) -> dict:
+    """Dual post-order trees (host only): parent, child0, child1, dual, depth."""
+    out = {k: np.zeros(p, np.int32) for k in ("parent", "child0", "child1",
+                                               "dual", "depth")}
+    _check(lib().dpdr_tree(p, *[out[k].ctypes.data_as(_IP) for k in
+                                ("parent", "child0", "child1", "dual",
+                                 "depth")]), "dpdr_tree")
+    return out
+
+
+def blocks(m: int, b: int) -> np.ndarray:
+    s = np.zeros(b + 1, np.int64)
+    _check(lib().dpdr_blocks(m, b, s.ctypes.data_as(_I64P)), "dpdr_blocks")
+    return s
+
+
+def block_count_rule(p: int, m: int, kappa: float = 0.0) -> int:
+    b = lib().dpdr_block_count_rule(p, m, kappa)
+    if b < 1:
+        raise DpdrError(lib().dpdr_last_error(), "dpdr_block_count_rule")
+    return b
+
+
+def _addr(t) -> int:
+    if isinstance(t, int):
+        return t
+    return int(t.data_ptr())
+
+
+def _ptr_array(ts: Sequence) -> ctypes.Array:
+    arr = (ctypes.c_void_p * len(ts))()
+    for i, t in enumerate(ts):
+        arr[i] = _addr(t)
+    return arr
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        import torch
+        return int(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return stream
+    return int(stream.cuda_stream)
+
+
+DTYPES = {"int32": DPDR_INT32, "float32": DPDR_FLOAT32,
+          "mat2x2u32": DPDR_MAT2X2_U32}
+
+
+class Plan:
+    """A plan for p virtual ranks of m elements (``dpdr_plan``)."""
+
+    def __init__(self, p: int, m: int, dtype, b: int = 0):
+        dt = DTYPES[dtype] if isinstance(dtype, str) else int(dtype)
+        op = DPDR_OP_MATMUL if dt == DPDR_MAT2X2_U32 else DPDR_OP_SUM
+        L = lib()
+        h = L.dpdr_plan(int(p), int(m), dt, op, int(b))
+        if not h:
+            raise DpdrError(L.dpdr_last_error(), "dpdr_plan")
+        self._h = h
+        self.p, self.m, self.dtype = int(p), int(m), dt
+
+    def close(self) -> None:
+        if getattr(self, "_h", None):
+            lib().dpdr_plan_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    # ---------------------------------------------------------------- facts
+    def query(self) -> dict:
+        out = {k: np.zeros(self.p, np.int32) for k in ("parent", "child0",
+                                                        "child1", "dual",
+                                                        "depth")}
+        b = ctypes.c_int(0)
+        _check(lib().dpdr_plan_query(self._h, *[out[k].ctypes.data_as(_IP) for k in
+                                                 ("parent", "child0", "child1",
+                                                  "dual", "depth")],
+                                     ctypes.byref(b)), "dpdr_plan_query")
+        out["b"] = b.value
+        return out
+
+    def info(self) -> dict:
+        v = np.zeros(9, np.int64)
+        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), 9),
+               "dpdr_plan_info")
+        keys = ("p", "m", "b", "max_depth", "auto_mode", "sched_ctas",
+                "sched_ranks_per_cta", "scratch_bytes", "vector_path")
+        return {k: int(x) for k, x in zip(keys, v)}
+
+    def set(self, key: int, value: int) -> None:
+        _check(lib().dpdr_plan_set(self._h, int(key), int(value)), "dpdr_plan_set")
+
+    # ------------------------------------------------------------------ run
+    def allreduce(self, xs: Sequence, ys: Sequence, stream=None) -> None:
+        """Fused kernel: every ys[i] <- x_0 (.) ... (.) x_{p-1}."""
+        assert len(xs) == self.p and len(ys) == self.p
+        _check(lib().dpdr_allreduce(self._h, _ptr_array(xs), _ptr_array(ys),
+                                    _stream(stream)), "dpdr_allreduce")
+
+    def allreduce_schedule(self, xs: Sequence, ys: Sequence, stream=None) -> None:
+        """Schedule-faithful kernel (Algorithm 1 round by round)."""
+        assert len(xs) == self.p and len(ys) == self.p
+        _check(lib().dpdr_allreduce_schedule(self._h, _ptr_array(xs),
+                                             _ptr_array(ys), _stream(stream)),
+               "dpdr_allreduce_schedule")
+
+    def allreduce_host(self, xh: Sequence, yh: Sequence, xd: Sequence,
+                       yd: Sequence, stream=None) -> None:
+        """Host buffers in and out, device buffers as staging."""
+        _check(lib().dpdr_allreduce_host(self._h, _ptr_array(xh), _ptr_array(yh),
+                                         _ptr_array(xd), _ptr_array(yd),
+                                         _stream(stream)), "dpdr_allreduce_host")
+
+    def sync(self, stream=None) -> None:
+        """Wait for the stream; raise DpdrError on a schedule-kernel timeout."""
+        _check(lib().dpdr_plan_sync(self._h, _stream(stream)), "dpdr_plan_sync")

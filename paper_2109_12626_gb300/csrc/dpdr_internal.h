@@ -1,0 +1,102 @@
+// dpdr_internal.h -- plan layout shared by the host code and the two kernel
+// launchers of the library (not part of the public ABI).
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "../../include/dpdr.h"
+
+namespace dpdr {
+
+// Tape byte of the column-streaming fold, one per rank in post-order:
+//   bits 0-1  number of children c in {0,1,2}
+//   bit  2    keep: the node value is parked in slot d (the node is the
+//             child_1 of its parent, or the lower root r0)
+//   bits 3-7  depth d
+constexpr int kTapeKeep = 4;
+constexpr int kMaxDepth = 31;
+
+// Entries of the level table of the shared-memory tile fold: internal
+// nodes, deepest level first, as (node, child_1 or -1); child_0 = node-1.
+struct LevelNode {
+    int node;
+    int child1;
+};
+
+struct Plan {
+    int p = 0;
+    int64_t m = 0;
+    int dtype = 0;
+    int op = 0;
+    int b = 1;
+    size_t esize = 4;
+    int device = 0;
+    int num_sms = 0;
+
+    // trees (Sec. 1.1)
+    std::vector<int> parent, child0, child1, dual, depth;
+    int max_depth = 0;
+    int r0 = -1, r1 = 0;
+    std::vector<uint8_t> tape;                 // column-streaming fold
+    std::vector<LevelNode> levels;             // tile fold
+    std::vector<int> level_off;                // nlevels + 1
+
+    // options
+    int fused_mode = 0;        // 0 auto, 1 stream, 2 tile
+    int64_t wait_ns = 4000000000LL;
+    int skip_rank = -1;
+    int sched_threads = 128;
+    int sched_rpc = 0;         // ranks per CTA, 0 = auto
+
+    // device memory: one allocation carved into the tables below
+    char* dmem = nullptr;
+    size_t dmem_bytes = 0;
+    const char** d_x = nullptr;      // [p] rank input pointers, then
+    char** d_y = nullptr;            // [p] rank output pointers (d_x + p)
+    uint8_t* d_tape = nullptr;       // [p rounded up to 8]
+    LevelNode* d_levels = nullptr;
+    int* d_level_off = nullptr;
+    int* d_tables = nullptr;         // parent, child0, child1, depth: 4 x [p]
+    uint32_t* d_ctrl = nullptr;      // up[p], down[p], abort word
+    uint32_t* d_err = nullptr;       // 4 words: status, rank, round, step
+    char* d_ring = nullptr;          // dual-root exchange slots: [2][2][slot]
+    size_t ring_slot_bytes = 0;
+    int* d_cta_first = nullptr;      // schedule CTA -> first rank (+1 entry)
+    int cta_capacity = 0;            // entries reserved in d_cta_first
+
+    // rank-pointer staging (pinned host), copied to d_x / d_y when they change
+    const void** h_ptrs = nullptr;   // [2p]
+    std::vector<const void*> last_x, last_y;
+    cudaEvent_t staged = nullptr;
+    bool staged_pending = false;     // d_x / d_y hold last_x / last_y
+
+    // facts
+    int last_vector_path = 0;
+    int sched_ctas = 0, sched_ranks_per_cta = 0;
+};
+
+// host-side builders (plan.cpp)
+void build_tree(int p, int* parent, int* child0, int* child1, int* dual,
+                int* depth);
+int block_count_rule(int p, int64_t m, double kappa);
+
+// errors (plan.cpp)
+int fail(int status, const std::string& msg);
+int cuda_fail(cudaError_t e, const char* what);
+
+// rank-pointer upload (api.cpp)
+int stage_pointers(Plan* P, const void* const* x, const void* const* y,
+                   cudaStream_t s);
+
+// launchers
+int fused_launch(Plan* P, cudaStream_t s);      // fused.cu
+int fused_auto_mode(const Plan* P);             // fused.cu
+int schedule_launch(Plan* P, cudaStream_t s);   // schedule.cu
+int schedule_configure(Plan* P);                // schedule.cu
+
+}  // namespace dpdr

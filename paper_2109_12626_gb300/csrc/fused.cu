@@ -1,0 +1,303 @@
+// fused.cu -- the fused bandwidth kernel of dpdr_allreduce.
+//
+// One launch computes y = v(r0) (.) v(r1) with the post-order bracketing of
+// Sec. 1.1 (v(i) = v(child_1) (.) (v(child_0) (.) x_i), child_0 = i-1) for
+// every element column and stores it to all p outputs.  Every input element
+// is read once and every output element written once: 2 p m element
+// transfers, the floor for any reduction-to-all whose p inputs and p outputs
+// live in device memory.  The tree's pipeline blocks (Algorithm 1) do not
+// change the result, so this kernel tiles by columns only.
+//
+// Two layouts of the same computation:
+//  * column streaming: one thread owns one 16-byte column unit and walks the
+//    p ranks in post-order, folding them with a register accumulator and a
+//    per-depth slot array in shared memory (the running post-order fold:
+//    a node's child_0 is the rank just before it and arrives in the
+//    accumulator; its child_1 value was parked in slot depth+1).  Eight
+//    ranks are loaded ahead of the fold.  Suits m >> p.
+//  * shared-memory tile: one CTA loads a tile of WU column units from all p
+//    ranks into shared memory with cp.async, evaluates the tree level by
+//    level (deepest first; all nodes of a level in parallel), then writes
+//    the result row to all p outputs.  Suits small m with large p, where
+//    column streaming would leave most SMs idle.
+#include <algorithm>
+
+#include "dpdr_internal.h"
+#include "ops.cuh"
+
+namespace dpdr {
+namespace {
+
+constexpr int kStreamThreads = 256;
+constexpr int kStreamAhead = 8;  // ranks loaded ahead (tape read 8 at a time)
+constexpr int kTileThreads = 256;
+constexpr size_t kTileSmemTarget = 96 * 1024;
+
+struct FusedArgs {
+    const char* const* x;   // [p] rank inputs
+    char* const* y;         // [p] rank outputs
+    const uint8_t* tape;    // [p rounded up to 8]
+    const LevelNode* levels;
+    const int* level_off;
+    int nlevels;
+    int p;
+    int r0, r1;
+    int64_t nvec;           // 16-byte units
+    int64_t nscalar;        // single elements after the vector units
+    int64_t scalar_base;    // element index of the first single element
+    int lg_wu;              // tile: log2 of vector units per row
+    int64_t vec_tiles;      // tile: number of vector tiles
+};
+
+template <class Op>
+struct VecUnit {
+    using T = uint4;
+    __device__ __forceinline__ static T ld(const char* row, int64_t u)
+    {
+        return ld_stream(row + u * 16);
+    }
+    __device__ __forceinline__ static void st(char* row, int64_t u, const T& v)
+    {
+        st_stream(row + u * 16, v);
+    }
+    __device__ __forceinline__ static T op(const T& a, const T& b) { return Op::vec(a, b); }
+};
+
+template <class Op>
+struct OneUnit {
+    using T = Elem<Op>;
+    __device__ __forceinline__ static T ld(const char* row, int64_t e)
+    {
+        return ld_one_stream<Op>(row + e * Op::kEsize);
+    }
+    __device__ __forceinline__ static void st(char* row, int64_t e, const T& v)
+    {
+        st_one_stream<Op>(row + e * Op::kEsize, v);
+    }
+    __device__ __forceinline__ static T op(const T& a, const T& b) { return comb<Op>(a, b); }
+};
+
+__device__ __forceinline__ const char* rank_ptr(const char* const* t, int i)
+{
+    return reinterpret_cast<const char*>(__ldg(reinterpret_cast<const unsigned long long*>(t) + i));
+}
+__device__ __forceinline__ char* rank_ptr_w(char* const* t, int i)
+{
+    return reinterpret_cast<char*>(__ldg(reinterpret_cast<const unsigned long long*>(t) + i));
+}
+
+// ---------------------------------------------------------------- streaming
+template <class U>
+__device__ __forceinline__ void stream_column(const FusedArgs& a, int64_t u,
+                                              typename U::T* slot, int stride)
+{
+    using T = typename U::T;
+    const int p = a.p;
+    T cur[kStreamAhead], nxt[kStreamAhead];
+#pragma unroll
+    for (int k = 0; k < kStreamAhead; k++)
+        if (k < p) cur[k] = U::ld(rank_ptr(a.x, k), u);
+    T acc = cur[0];
+    for (int i0 = 0; i0 < p; i0 += kStreamAhead) {
+#pragma unroll
+        for (int k = 0; k < kStreamAhead; k++)
+            if (i0 + kStreamAhead + k < p)
+                nxt[k] = U::ld(rank_ptr(a.x, i0 + kStreamAhead + k), u);
+        const unsigned long long tp =
+            __ldg(reinterpret_cast<const unsigned long long*>(a.tape + i0));
+#pragma unroll
+        for (int k = 0; k < kStreamAhead; k++) {
+            if (i0 + k < p) {
+                const unsigned t = unsigned(tp >> (8 * k)) & 0xffu;
+                const unsigned c = t & 3u, d = t >> 3;
+                T v = cur[k];
+                if (c >= 1) v = U::op(acc, v);                     // v(c0) (.) x_i
+                if (c == 2) v = U::op(slot[(d + 1) * stride], v);  // v(c1) (.) (..)
+                if (t & kTapeKeep) slot[d * stride] = v;
+                acc = v;
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kStreamAhead; k++) cur[k] = nxt[k];
+    }
+    const T y = (p >= 2) ? U::op(slot[0], acc) : acc;  // v(r0) (.) v(r1)
+#pragma unroll 4
+    for (int i = 0; i < p; i++) U::st(rank_ptr_w(a.y, i), u, y);
+}
+
+template <class Op>
+__global__ void __launch_bounds__(kStreamThreads, 3)
+fused_stream_kernel(FusedArgs a)
+{
+    extern __shared__ uint4 smem[];
+    const int64_t u = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (u < a.nvec) {
+        stream_column<VecUnit<Op>>(a, u, smem + threadIdx.x, blockDim.x);
+    } else if (u < a.nvec + a.nscalar) {
+        auto* slot = reinterpret_cast<Elem<Op>*>(smem) + threadIdx.x;
+        stream_column<OneUnit<Op>>(a, a.scalar_base + (u - a.nvec), slot, blockDim.x);
+    }
+}
+
+// --------------------------------------------------------------------- tile
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem)
+{
+    const unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all()
+{
+    asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;\n" ::: "memory");
+}
+
+// rows of WU units: row i < p holds rank i's tile, row p the result
+template <class U, bool kAsync>
+__device__ __forceinline__ void tile_body(const FusedArgs& a, int64_t u0,
+                                          int wu, int lg_wu, typename U::T* tile)
+{
+    using T = typename U::T;
+    const int p = a.p, tid = threadIdx.x, bd = blockDim.x;
+    const int WU = 1 << lg_wu;
+    const int n = p << lg_wu;
+    for (int idx = tid; idx < n; idx += bd) {
+        const int i = idx >> lg_wu, c = idx & (WU - 1);
+        if (c < wu) {
+            if constexpr (kAsync)
+                cp_async16(&tile[idx], rank_ptr(a.x, i) + (u0 + c) * 16);
+            else
+                tile[idx] = U::ld(rank_ptr(a.x, i), u0 + c);
+        }
+    }
+    if constexpr (kAsync) cp_async_wait_all();
+    __syncthreads();
+    for (int l = 0; l < a.nlevels; l++) {
+        const int beg = __ldg(a.level_off + l), end = __ldg(a.level_off + l + 1);
+        const int cnt = (end - beg) << lg_wu;
+        for (int idx = tid; idx < cnt; idx += bd) {
+            const int k = idx >> lg_wu, c = idx & (WU - 1);
+            if (c >= wu) continue;
+            const int node = __ldg(&a.levels[beg + k].node);
+            const int c1 = __ldg(&a.levels[beg + k].child1);
+            T v = U::op(tile[((node - 1) << lg_wu) + c], tile[(node << lg_wu) + c]);
+            if (c1 >= 0) v = U::op(tile[(c1 << lg_wu) + c], v);
+            tile[(node << lg_wu) + c] = v;
+        }
+        __syncthreads();
+    }
+    for (int c = tid; c < wu; c += bd) {
+        const T v1 = tile[(a.r1 << lg_wu) + c];
+        tile[(p << lg_wu) + c] = (p >= 2) ? U::op(tile[(a.r0 << lg_wu) + c], v1) : v1;
+    }
+    __syncthreads();
+    for (int idx = tid; idx < n; idx += bd) {
+        const int i = idx >> lg_wu, c = idx & (WU - 1);
+        if (c < wu) U::st(rank_ptr_w(a.y, i), u0 + c, tile[(p << lg_wu) + c]);
+    }
+}
+
+template <class Op>
+__global__ void __launch_bounds__(kTileThreads)
+fused_tile_kernel(FusedArgs a)
+{
+    extern __shared__ uint4 smem[];
+    const int64_t t = blockIdx.x;
+    if (t < a.vec_tiles) {
+        const int64_t u0 = t << a.lg_wu;
+        const int wu = int(lmin(int64_t(1) << a.lg_wu, a.nvec - u0));
+        tile_body<VecUnit<Op>, true>(a, u0, wu, a.lg_wu, smem);
+    } else {
+        // single elements: a row of a tile holds as many bytes as in the
+        // vector tiles, i.e. 16/esize times more units
+        const int lg = a.lg_wu + (Op::kEsize == 4 ? 2 : 0);
+        const int64_t e0 = (t - a.vec_tiles) << lg;
+        const int wu = int(lmin(int64_t(1) << lg, a.nscalar - e0));
+        tile_body<OneUnit<Op>, false>(a, a.scalar_base + e0, wu, lg,
+                                      reinterpret_cast<Elem<Op>*>(smem));
+    }
+}
+
+// --------------------------------------------------------------------- host
+template <class Op>
+int launch(Plan* P, FusedArgs a, int mode, cudaStream_t s)
+{
+    if (mode == 1) {
+        const int64_t units = a.nvec + a.nscalar;
+        const int64_t blocks = (units + kStreamThreads - 1) / kStreamThreads;
+        const size_t smem = size_t(P->max_depth + 1) * kStreamThreads * sizeof(uint4);
+        if (blocks > 0x7fffffff) return fail(DPDR_ERR_INVALID, "m too large");
+        cudaError_t e = cudaFuncSetAttribute(fused_stream_kernel<Op>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             int(smem));
+        if (e != cudaSuccess) return cuda_fail(e, "fused stream attribute");
+        fused_stream_kernel<Op><<<unsigned(blocks), kStreamThreads, smem, s>>>(a);
+    } else {
+        const size_t smem = size_t(P->p + 1) * (size_t(16) << a.lg_wu);
+        const int64_t lg_s = a.lg_wu + (Op::kEsize == 4 ? 2 : 0);
+        const int64_t scal_tiles = (a.nscalar + (int64_t(1) << lg_s) - 1) >> lg_s;
+        const int64_t blocks = a.vec_tiles + scal_tiles;
+        if (blocks > 0x7fffffff) return fail(DPDR_ERR_INVALID, "m too large");
+        cudaError_t e = cudaFuncSetAttribute(fused_tile_kernel<Op>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             int(smem));
+        if (e != cudaSuccess) return cuda_fail(e, "fused tile attribute");
+        fused_tile_kernel<Op><<<unsigned(blocks), kTileThreads, smem, s>>>(a);
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "fused kernel launch");
+    return DPDR_OK;
+}
+
+// largest power-of-two vector units per tile row that fits the smem target
+int tile_lg_wu(const Plan* P)
+{
+    const size_t row = size_t(P->p + 1) * 16;
+    if (row > 200 * 1024) return -1;  // not even one unit per row fits
+    int lg = 0;
+    while (lg < 6 && row * (size_t(2) << lg) <= kTileSmemTarget) lg++;
+    return lg;
+}
+
+}  // namespace
+
+int fused_auto_mode(const Plan* P)
+{
+    if (tile_lg_wu(P) < 0) return 1;
+    const int64_t units = P->m * int64_t(P->esize) / 16;
+    // column streaming needs enough independent columns to fill every SM
+    return units >= int64_t(P->num_sms) * 1024 ? 1 : 2;
+}
+
+int fused_launch(Plan* P, cudaStream_t s)
+{
+    if (P->m == 0) return DPDR_OK;
+    int mode = P->fused_mode ? P->fused_mode : fused_auto_mode(P);
+    const int lg = tile_lg_wu(P);
+    if (mode == 2 && lg < 0) return fail(DPDR_ERR_INVALID, "tile mode: p too large");
+
+    FusedArgs a;
+    a.x = P->d_x;
+    a.y = P->d_y;
+    a.tape = P->d_tape;
+    a.levels = P->d_levels;
+    a.level_off = P->d_level_off;
+    a.nlevels = int(P->level_off.size()) - 1;
+    a.p = P->p;
+    a.r0 = P->r0;
+    a.r1 = P->r1;
+    const bool vec = P->last_vector_path != 0;
+    const int epv = int(16 / P->esize);
+    a.nvec = vec ? P->m / epv : 0;
+    a.scalar_base = a.nvec * epv;
+    a.nscalar = P->m - a.scalar_base;
+    a.lg_wu = lg < 0 ? 0 : lg;
+    a.vec_tiles = (a.nvec + (int64_t(1) << a.lg_wu) - 1) >> a.lg_wu;
+
+    switch (P->dtype) {
+    case DPDR_INT32: return launch<SumI32>(P, a, mode, s);
+    case DPDR_FLOAT32: return launch<SumF32>(P, a, mode, s);
+    default: return launch<MatU32>(P, a, mode, s);
+    }
+}
+
+}  // namespace dpdr

@@ -1,0 +1,369 @@
+// schedule.cu -- the schedule-faithful persistent kernel of
+// dpdr_allreduce_schedule: Algorithm 1 run by every virtual rank.
+//
+// Rank i runs rounds j = 0..b+d_i (d_i = depth).  Each round has the three
+// bidirectional steps of Algorithm 1, in order:
+//   child_0 : send final Y[j-(d_i+1)], receive the child's partial Y[j] into
+//             t and form Y[j] = t (.) Y[j]
+//   child_1 : the same with the second child
+//   dual    : (roots) send the partial Y[j], receive the dual's partial t;
+//             the lower root forms Y[j] (.) t, the higher t (.) Y[j]
+//   parent  : (others) send the partial Y[j], receive final Y[j-d_i]
+// Blocks outside [0,b) are empty; an exchange empty both ways is skipped.
+//
+// On one GPU an exchange is a pair of published blocks in device memory.
+// Every rank owns two monotone counters: up[i] = number of partial blocks it
+// has published, down[i] = number of final blocks it holds.  A send is a
+// release store of the counter after the block is written; a receive is an
+// acquire load of the partner's counter followed by reading the partner's
+// block straight from the partner's buffer (L2-coherent loads), fused with
+// the (.) -- the temporary t of Algorithm 1 never materialises.  Where a
+// partial lives: a leaf's partial block j is x_i[j] itself, an inner node's
+// is y_i[j], a root's is one of two exchange slots per root (the dual reads
+// it while the root overwrites y_r[j] with the final block).  A child
+// overwrites its partial y_c[k] with the final block only after its parent
+// published final block k, which the parent does after it consumed partial
+// k: the data dependencies of the algorithm order every reuse, so a sender
+// never waits for its receiver.
+//
+// CTAs own contiguous rank ranges that never straddle the two trees and run
+// their ranks in increasing order inside each round.  Every wait is then on
+// a lower rank of the same round, on an earlier round, or (r0 only) on the
+// dual r1 whose partial depends on tree 1 alone, so with all CTAs resident
+// (cooperative launch) the schedule cannot deadlock.  Each wait is bounded
+// in time; an expired wait records {rank, round, step} in the plan's error
+// word, raises an abort flag that ends every other wait, and returns.
+#include <algorithm>
+
+#include "dpdr_internal.h"
+#include "ops.cuh"
+
+namespace dpdr {
+namespace {
+
+constexpr int kSchedMaxThreads = 256;
+
+struct SchedArgs {
+    const char* const* x;
+    char* const* y;
+    const int* parent;
+    const int* child0;
+    const int* child1;
+    const int* depth;
+    const int* cta_first;
+    uint32_t* up;
+    uint32_t* down;
+    uint32_t* abort_flag;
+    uint32_t* err;
+    char* ring;
+    int64_t ring_slot;
+    int p, b, r0, r1;
+    int64_t m, q, rem;
+    int64_t wait_ns;
+    int skip_rank;
+    int vec;
+};
+
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p)
+{
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_release(uint32_t* p, uint32_t v)
+{
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ uint32_t ld_relaxed(const uint32_t* p)
+{
+    uint32_t v;
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ uint64_t now_ns()
+{
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ int64_t blk_start(const SchedArgs& a, int j)
+{
+    return int64_t(j) * a.q + lmin(j, a.rem);
+}
+
+// Thread 0 waits for *ctr >= target within the plan's time bound; the CTA
+// learns the outcome through shared memory.  Returns false on timeout or
+// abort (then the caller returns from the kernel).
+__device__ __forceinline__ bool cta_wait(const SchedArgs& a, const uint32_t* ctr, uint32_t target,
+                         int rank, int j, int step)
+{
+    __shared__ int ok;
+    if (threadIdx.x == 0) {
+        int r = 1;
+        if (ld_acquire(ctr) < target) {
+            const uint64_t t0 = now_ns();
+            unsigned sleep = 32;
+            while (true) {
+                if (ld_acquire(ctr) >= target) break;
+                if (ld_relaxed(a.abort_flag)) { r = 0; break; }
+                if (now_ns() - t0 > uint64_t(a.wait_ns)) {
+                    if (atomicCAS(a.err, 0u, uint32_t(DPDR_ERR_TIMEOUT)) == 0u) {
+                        a.err[1] = uint32_t(rank);
+                        a.err[2] = uint32_t(j);
+                        a.err[3] = uint32_t(step);
+                    }
+                    __threadfence();
+                    atomicExch(a.abort_flag, 1u);
+                    r = 0;
+                    break;
+                }
+                __nanosleep(sleep);
+                if (sleep < 1024) sleep <<= 1;
+            }
+        }
+        ok = r;
+    }
+    __syncthreads();
+    const int r = ok;
+    __syncthreads();
+    return r != 0;
+}
+
+// Release the CTA's writes to the rank's partner(s).
+__device__ __forceinline__ void publish(const SchedArgs& a, uint32_t* ctr, uint32_t v, int rank)
+{
+    __syncthreads();
+    if (threadIdx.x == 0 && rank != a.skip_rank) {
+        __threadfence();
+        st_release(ctr, v);
+    }
+}
+
+// dst[k] = lo[k] (.) hi[k] for k in [s, e); rows are virtual bases indexed
+// by global element number.  dst may equal hi.  With lo == nullptr it is a
+// plain copy dst[k] = hi[k].
+template <class Op>
+__device__ __forceinline__ void block_op(const SchedArgs& a, char* dst, const char* lo,
+                         const char* hi, int64_t s, int64_t e)
+{
+    constexpr int EPV = Op::kEpv;
+    constexpr int ES = Op::kEsize;
+    const int tid = threadIdx.x, bd = blockDim.x;
+    int64_t vs = 0, ve = 0;
+    if (a.vec) {
+        vs = (s + EPV - 1) / EPV;
+        ve = e / EPV;
+        if (vs > ve) vs = ve = 0;
+    }
+    // single elements: the unaligned head and tail around the vector range
+    int64_t head_end = e, tail_beg = e;
+    if (vs < ve) {
+        head_end = vs * EPV;
+        tail_beg = ve * EPV;
+    }
+    for (int pass = 0; pass < 2; pass++) {
+        const int64_t b0 = pass ? tail_beg : s, b1 = pass ? e : head_end;
+        for (int64_t k = b0 + tid; k < b1; k += bd) {
+            const Elem<Op> h = ld_one_l2<Op>(hi + k * ES);
+            st_one_l2<Op>(dst + k * ES, lo ? comb<Op>(ld_one_l2<Op>(lo + k * ES), h) : h);
+        }
+    }
+    // 16-byte units, four in flight per thread
+    constexpr int B = 4;
+    for (int64_t v0 = vs + tid; v0 < ve; v0 += int64_t(B) * bd) {
+        uint4 hv[B], lv[B];
+#pragma unroll
+        for (int t = 0; t < B; t++) {
+            const int64_t v = v0 + int64_t(t) * bd;
+            if (v < ve) {
+                hv[t] = ld_l2(hi + v * 16);
+                if (lo) lv[t] = ld_l2(lo + v * 16);
+            }
+        }
+#pragma unroll
+        for (int t = 0; t < B; t++) {
+            const int64_t v = v0 + int64_t(t) * bd;
+            if (v < ve) st_l2(dst + v * 16, lo ? Op::vec(lv[t], hv[t]) : hv[t]);
+        }
+    }
+}
+
+__device__ __forceinline__ char* ring_base(const SchedArgs& a, int side, int j,
+                                           int64_t s, int epv, int es)
+{
+    char* slot = a.ring + (int64_t(side) * 2 + (j & 1)) * a.ring_slot;
+    return slot - (s - s % epv) * es;  // keeps element k congruent mod 16
+}
+
+template <class Op>
+__device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j)
+{
+    const int d = __ldg(a.depth + i);
+    const int c0 = __ldg(a.child0 + i), c1 = __ldg(a.child1 + i);
+    const int par = __ldg(a.parent + i);
+    const char* xi = reinterpret_cast<const char*>(__ldg(reinterpret_cast<const unsigned long long*>(a.x) + i));
+    char* yi = reinterpret_cast<char*>(__ldg(reinterpret_cast<const unsigned long long*>(a.y) + i));
+    const bool root = par < 0;
+    const bool paired_root = root && a.p >= 2;
+    const bool inb = j < a.b;
+    const int64_t s = inb ? blk_start(a, j) : 0, e = inb ? blk_start(a, j + 1) : 0;
+    const int side = (i == a.r0) ? 0 : 1;
+    char* dst = paired_root ? ring_base(a, side, j, s, Op::kEpv, Op::kEsize) : yi;
+
+    // steps 1 and 2: child_0 then child_1; the send half (final block
+    // j-(d+1)) is read by the child itself from y_i once down[i] covers it
+    bool have = false;
+    for (int k = 0; k < 2; k++) {
+        const int c = k ? c1 : c0;
+        if (c < 0 || !inb) continue;
+        if (!cta_wait(a, a.up + c, uint32_t(j + 1), i, j, k)) return false;
+        const bool leaf = __ldg(a.child0 + c) < 0;
+        const char* src = leaf
+            ? reinterpret_cast<const char*>(__ldg(reinterpret_cast<const unsigned long long*>(a.x) + c))
+            : reinterpret_cast<const char*>(__ldg(reinterpret_cast<const unsigned long long*>(a.y) + c));
+        block_op<Op>(a, dst, src, have ? dst : xi, s, e);  // Y[j] = t (.) Y[j]
+        have = true;
+        __syncthreads();
+    }
+
+    if (paired_root) {  // step 3 at a root: exchange partials with the dual
+        if (!inb) return true;
+        if (!have) {
+            block_op<Op>(a, dst, nullptr, xi, s, e);
+            __syncthreads();
+        }
+        publish(a, a.up + i, uint32_t(j + 1), i);
+        const int du = (i == a.r0) ? a.r1 : a.r0;
+        if (!cta_wait(a, a.up + du, uint32_t(j + 1), i, j, 2)) return false;
+        const char* other = ring_base(a, 1 - side, j, s, Op::kEpv, Op::kEsize);
+        if (i == a.r0)
+            block_op<Op>(a, yi, dst, other, s, e);  // lower root: Y[j] (.) t
+        else
+            block_op<Op>(a, yi, other, dst, s, e);  // higher root: t (.) Y[j]
+        publish(a, a.down + i, uint32_t(j + 1), i);
+        return true;
+    }
+    if (root) {  // p == 1: one processor, y = x
+        if (inb && xi != yi) {
+            block_op<Op>(a, yi, nullptr, xi, s, e);
+            __syncthreads();
+        }
+        return true;
+    }
+    // step 3 elsewhere: partial Y[j] up (in y_i, or x_i for a leaf), final
+    // Y[j-d] down from the parent
+    if (inb) publish(a, a.up + i, uint32_t(j + 1), i);
+    const int kf = j - d;
+    if (kf >= 0 && kf < a.b) {
+        if (!cta_wait(a, a.down + par, uint32_t(kf + 1), i, j, 3)) return false;
+        const char* yp = reinterpret_cast<const char*>(__ldg(reinterpret_cast<const unsigned long long*>(a.y) + par));
+        block_op<Op>(a, yi, nullptr, yp, blk_start(a, kf), blk_start(a, kf + 1));
+        publish(a, a.down + i, uint32_t(kf + 1), i);
+    }
+    return true;
+}
+
+template <class Op>
+__global__ void __launch_bounds__(kSchedMaxThreads, 4) schedule_kernel(SchedArgs a)
+{
+    const int first = __ldg(a.cta_first + blockIdx.x);
+    const int last = __ldg(a.cta_first + blockIdx.x + 1);
+    int rounds = 0;
+    for (int i = first; i < last; i++) rounds = max(rounds, a.b + __ldg(a.depth + i));
+    for (int j = 0; j <= rounds; j++) {
+        for (int i = first; i < last; i++) {
+            if (j > a.b + __ldg(a.depth + i)) continue;
+            if (!run_round<Op>(a, i, j)) return;
+        }
+    }
+}
+
+template <class Op>
+const void* kernel_ptr()
+{
+    return reinterpret_cast<const void*>(&schedule_kernel<Op>);
+}
+
+const void* kernel_for(int dtype)
+{
+    switch (dtype) {
+    case DPDR_INT32: return kernel_ptr<SumI32>();
+    case DPDR_FLOAT32: return kernel_ptr<SumF32>();
+    default: return kernel_ptr<MatU32>();
+    }
+}
+
+}  // namespace
+
+// Choose ranks per CTA so that every CTA can be resident at once, with CTA
+// boundaries on the tree boundary, and upload the CTA -> rank table.
+int schedule_configure(Plan* P)
+{
+    int occ = 0;
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+        &occ, kernel_for(P->dtype), P->sched_threads, 0);
+    if (e != cudaSuccess) return cuda_fail(e, "schedule occupancy");
+    const int64_t kmax = int64_t(occ) * P->num_sms;
+    const int n0 = P->p / 2, n1 = P->p - n0;
+    auto ctas = [&](int r) { return (n0 + r - 1) / r + (n1 + r - 1) / r; };
+    int R = P->sched_rpc;
+    if (R == 0) {
+        R = 1;
+        while (R < P->p && ctas(R) > kmax) R++;
+    }
+    std::vector<int> first;
+    for (int lo = 0; lo < n0; lo += R) first.push_back(lo);
+    for (int lo = n0; lo < P->p; lo += R) first.push_back(lo);
+    first.push_back(P->p);
+    P->sched_ctas = int(first.size()) - 1;
+    P->sched_ranks_per_cta = R;
+    if (P->sched_ctas > P->cta_capacity) return fail(DPDR_ERR_INVALID, "too many CTAs");
+    e = cudaMemcpy(P->d_cta_first, first.data(), sizeof(int) * first.size(),
+                   cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "schedule table upload");
+    return DPDR_OK;
+}
+
+int schedule_launch(Plan* P, cudaStream_t s)
+{
+    if (P->m == 0) return DPDR_OK;
+    SchedArgs a;
+    a.x = P->d_x;
+    a.y = P->d_y;
+    a.parent = P->d_tables;
+    a.child0 = P->d_tables + P->p;
+    a.child1 = P->d_tables + 2 * P->p;
+    a.depth = P->d_tables + 3 * P->p;
+    a.cta_first = P->d_cta_first;
+    a.up = P->d_ctrl;
+    a.down = P->d_ctrl + P->p;
+    a.abort_flag = P->d_ctrl + 2 * P->p;
+    a.err = P->d_err;
+    a.ring = P->d_ring;
+    a.ring_slot = int64_t(P->ring_slot_bytes);
+    a.p = P->p;
+    a.b = P->b;
+    a.r0 = P->r0;
+    a.r1 = P->r1;
+    a.m = P->m;
+    a.q = P->m / P->b;
+    a.rem = P->m % P->b;
+    a.wait_ns = P->wait_ns;
+    a.skip_rank = P->skip_rank;
+    a.vec = P->last_vector_path;
+
+    cudaError_t e = cudaMemsetAsync(P->d_ctrl, 0, sizeof(uint32_t) * (2 * size_t(P->p) + 1), s);
+    if (e != cudaSuccess) return cuda_fail(e, "schedule counter reset");
+    void* args[] = {&a};
+    e = cudaLaunchCooperativeKernel(kernel_for(P->dtype), dim3(P->sched_ctas),
+                                    dim3(P->sched_threads), args, 0, s);
+    if (e == cudaErrorCooperativeLaunchTooLarge) {
+        cudaGetLastError();
+        return fail(DPDR_ERR_NOT_COOPERATIVE, "schedule kernel: CTAs cannot be co-resident");
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "schedule kernel launch");
+    return DPDR_OK;
+}
+
+}  // namespace dpdr

@@ -1,0 +1,233 @@
+"""GPU parity: both kernels of the C ABI against the CPU oracle, element by
+element and bit for bit (float32 included: every kernel keeps the dual-tree
+bracketing of Sec. 1.1 / Algorithm 1, so the bits must agree).
+
+Sizes are ones the oracle finishes in seconds but that span several tiles
+and a ragged tail; the edge cases are p = 1, 2, 3, m = 0 and 1, in-place
+buffers, 4-byte-aligned (not 16-byte) buffers, and every block count from 1
+to m."""
+import numpy as np
+import pytest
+import torch
+
+from gpu_util import bits, empty_like_ranks, expect_bits, host_inputs, to_device
+
+pytestmark = pytest.mark.gpu
+
+LOHI3 = dict(lo=-(1 << 20), hi=1 << 20)
+CASES = [
+    # id, kind, seed, p, m, kwargs, schedule block counts
+    ("p7_m1000_int32", "int32", 1, 7, 1000, dict(lo=-1000, hi=1000), [4, 1, 3, 1000]),
+    ("p36_m65536_mat", "mat2x2u32", 2, 36, 65536, {}, [16, 1, 5]),
+    ("p1152_m1_int32", "int32", 3, 1152, 1, LOHI3, [1]),
+    ("p1152_m3_int32", "int32", 3, 1152, 3, LOHI3, [1, 3]),
+    ("p1152_m4099_int32", "int32", 3, 1152, 4099, LOHI3, [1, 4, 16, 64]),
+    ("p1152_m4099_f32", "float32", 4, 1152, 4099, dict(sigma=1.0), [7, 0]),
+    ("p32_m65541_f32", "float32", 5, 32, 65541, dict(sigma=1e-3), [64, 256]),
+    ("p32_m300000_f32", "float32", 5, 32, 300000, dict(sigma=1e-3), [1024]),
+    ("p1_m17_f32", "float32", 6, 1, 17, {}, [1, 5]),
+    ("p2_m333_f32", "float32", 6, 2, 333, {}, [1, 2, 333]),
+    ("p3_m10_mat", "mat2x2u32", 6, 3, 10, {}, [1, 10]),
+    ("p5_m1_int32", "int32", 6, 5, 1, dict(lo=-5, hi=5), [1]),
+    ("p100_m77_mat", "mat2x2u32", 7, 100, 77, {}, [1, 7, 77]),
+    ("p255_m2050_f32", "float32", 8, 255, 2050, {}, [3, 16]),
+]
+
+
+@pytest.fixture(scope="module")
+def pkg():
+    from paper_2109_12626_gb300 import build as B
+    B.build()
+    import paper_2109_12626_gb300 as P
+    return P
+
+
+def _want(orc, x, kind):
+    dt = {"int32": orc.I32, "float32": orc.F32, "mat2x2u32": orc.MAT}[kind]
+    return expect_bits(orc.tree_fold(x, dt))
+
+
+def _check_all(ys, want, guards=None):
+    for i, y in enumerate(ys):
+        got = bits(y)
+        assert got.shape == want.shape
+        bad = np.nonzero(got != want)[0]
+        assert bad.size == 0, "rank %d: %d mismatches, first at %d" % (i, bad.size, bad[0])
+
+
+@pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
+@pytest.mark.parametrize("mode", [1, 2], ids=["stream", "tile"])
+def test_fused_matches_oracle(pkg, orc, case, mode):
+    _, kind, seed, p, m, kw, _ = case
+    dev = torch.device("cuda:0")
+    x = host_inputs(kind, seed, p, m, **kw)
+    want = _want(orc, x, kind)
+    xs, _ = to_device(x, kind, dev)
+    ys, _ = empty_like_ranks(xs)
+    with pkg.Plan(p, m, kind, 4) as plan:
+        plan.set(pkg.OPT_FUSED_MODE, mode)
+        plan.allreduce(xs, ys)
+        plan.sync()
+        assert plan.info()["vector_path"] == 1
+    _check_all(ys, want)
+    for i in range(p):  # inputs untouched
+        assert np.array_equal(bits(xs[i]), expect_bits(x[i]))
+
+
+@pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
+def test_schedule_matches_oracle(pkg, orc, case):
+    _, kind, seed, p, m, kw, blist = case
+    dev = torch.device("cuda:0")
+    x = host_inputs(kind, seed, p, m, **kw)
+    want = _want(orc, x, kind)
+    xs, _ = to_device(x, kind, dev)
+    for b in blist:
+        ys, _ = empty_like_ranks(xs)
+        with pkg.Plan(p, m, kind, b) as plan:
+            plan.allreduce_schedule(xs, ys)
+            plan.sync()
+        _check_all(ys, want)
+    for i in range(p):
+        assert np.array_equal(bits(xs[i]), expect_bits(x[i]))
+
+
+@pytest.mark.parametrize("kind,p,m", [("int32", 7, 1000), ("float32", 1152, 4099),
+                                      ("mat2x2u32", 36, 999), ("float32", 2, 5)])
+@pytest.mark.parametrize("run", ["fused_stream", "fused_tile", "schedule"])
+def test_in_place(pkg, orc, kind, p, m, run):
+    """y[i] == x[i]: Algorithm 1 works in place (Y <- x_i, y ends in Y)."""
+    x = host_inputs(kind, 11, p, m)
+    want = _want(orc, x, kind)
+    xs, _ = to_device(x, kind, torch.device("cuda:0"))
+    with pkg.Plan(p, m, kind, 3) as plan:
+        if run == "schedule":
+            plan.allreduce_schedule(xs, xs)
+        else:
+            plan.set(pkg.OPT_FUSED_MODE, 1 if run == "fused_stream" else 2)
+            plan.allreduce(xs, xs)
+        plan.sync()
+    _check_all(xs, want)
+
+
+@pytest.mark.parametrize("kind,p,m", [("int32", 7, 1001), ("float32", 1152, 133),
+                                      ("mat2x2u32", 36, 257), ("float32", 32, 9999)])
+@pytest.mark.parametrize("run", ["fused_stream", "fused_tile", "schedule"])
+def test_four_byte_aligned_buffers(pkg, orc, kind, p, m, run):
+    """Buffers only 4-byte aligned take the single-element paths."""
+    x = host_inputs(kind, 12, p, m)
+    want = _want(orc, x, kind)
+    dev = torch.device("cuda:0")
+    xs, keep_x = to_device(x, kind, dev, pad_front=1)
+    ys, keep_y = empty_like_ranks(xs, pad_front=3)
+    with pkg.Plan(p, m, kind, 4) as plan:
+        if run == "schedule":
+            plan.allreduce_schedule(xs, ys)
+        else:
+            plan.set(pkg.OPT_FUSED_MODE, 1 if run == "fused_stream" else 2)
+            plan.allreduce(xs, ys)
+        plan.sync()
+        assert plan.info()["vector_path"] == 0
+    _check_all(ys, want)
+
+
+@pytest.mark.parametrize("run", ["fused_stream", "fused_tile", "schedule"])
+def test_guard_words_untouched(pkg, orc, run):
+    """No kernel writes past the m elements of an output."""
+    kind, p, m = "float32", 36, 4097
+    x = host_inputs(kind, 13, p, m)
+    want = _want(orc, x, kind)
+    dev = torch.device("cuda:0")
+    xs, _ = to_device(x, kind, dev)
+    bases = [torch.full((m + 64,), 7.25, device=dev) for _ in range(p)]
+    ys = [bb[:m] for bb in bases]
+    with pkg.Plan(p, m, kind, 5) as plan:
+        if run == "schedule":
+            plan.allreduce_schedule(xs, ys)
+        else:
+            plan.set(pkg.OPT_FUSED_MODE, 1 if run == "fused_stream" else 2)
+            plan.allreduce(xs, ys)
+        plan.sync()
+    _check_all(ys, want)
+    for bb in bases:
+        assert bool((bb[m:] == 7.25).all())
+
+
+def test_m_zero_is_a_no_op(pkg):
+    dev = torch.device("cuda:0")
+    xs = [torch.zeros(4, device=dev) for _ in range(5)]
+    ys = [torch.full((4,), 3.0, device=dev) for _ in range(5)]
+    with pkg.Plan(5, 0, "float32", 0) as plan:
+        assert plan.query()["b"] == 1
+        plan.allreduce(xs, ys)
+        plan.allreduce_schedule(xs, ys)
+        plan.sync()
+    assert all(bool((y == 3.0).all()) for y in ys)
+
+
+def test_repeated_calls_and_pointer_changes(pkg, orc):
+    """The rank-pointer table is re-staged when the buffers change."""
+    kind, p, m = "int32", 7, 1000
+    dev = torch.device("cuda:0")
+    with pkg.Plan(p, m, kind, 4) as plan:
+        for seed in (21, 22, 23):
+            x = host_inputs(kind, seed, p, m, lo=-1000, hi=1000)
+            want = _want(orc, x, kind)
+            xs, _ = to_device(x, kind, dev)
+            for _ in range(2):
+                ys, _ = empty_like_ranks(xs)
+                plan.allreduce(xs, ys)
+                _check_all(ys, want)
+                ys2, _ = empty_like_ranks(xs)
+                plan.allreduce_schedule(xs, ys2)
+                plan.sync()
+                _check_all(ys2, want)
+
+
+def test_host_buffers_end_to_end(pkg, orc):
+    kind, p, m = "float32", 32, 10007
+    x = host_inputs(kind, 31, p, m, sigma=1e-3)
+    want = _want(orc, x, kind)
+    dev = torch.device("cuda:0")
+    xh = [torch.from_numpy(x[i].copy()).pin_memory() for i in range(p)]
+    yh = [torch.zeros(m).pin_memory() for _ in range(p)]
+    xd = [torch.empty(m, device=dev) for _ in range(p)]
+    yd = [torch.empty(m, device=dev) for _ in range(p)]
+    with pkg.Plan(p, m, kind, 0) as plan:
+        plan.allreduce_host(xh, yh, xd, yd)
+        plan.sync()
+    _check_all(yh, want)
+
+
+def test_invalid_arguments(pkg):
+    from paper_2109_12626_gb300 import DpdrError, _native as N
+    dev = torch.device("cuda:0")
+    L = N.lib()
+    assert not L.dpdr_plan(0, 10, N.DPDR_INT32, N.DPDR_OP_SUM, 1)
+    assert L.dpdr_last_error() == N.DPDR_ERR_INVALID
+    assert not L.dpdr_plan(4, 10, N.DPDR_INT32, N.DPDR_OP_MATMUL, 1)
+    assert not L.dpdr_plan(4, -1, N.DPDR_FLOAT32, N.DPDR_OP_SUM, 1)
+    base = torch.zeros(4096, device=dev)
+    with pkg.Plan(3, 100, "float32", 1) as plan:
+        xs = [torch.zeros(100, device=dev) for _ in range(3)]
+        # two outputs overlapping
+        with pytest.raises(DpdrError) as e:
+            plan.allreduce(xs, [base[0:100], base[50:150], base[200:300]])
+        assert e.value.status == N.DPDR_ERR_INVALID
+        # an output overlapping another rank's input
+        with pytest.raises(DpdrError):
+            plan.allreduce([base[0:100], xs[1], xs[2]], [xs[0], base[1000:1100], base[40:140]])
+        # 2-byte misalignment
+        raw = torch.zeros(1000, dtype=torch.int16, device=dev)
+        with pytest.raises(DpdrError):
+            plan.allreduce([raw.data_ptr() + 2] + xs[1:], [base[0:100], base[200:300], base[400:500]])
+        # NULL buffer
+        with pytest.raises(DpdrError):
+            plan.allreduce([0] + xs[1:], [base[0:100], base[200:300], base[400:500]])
+        # the plan still works afterwards
+        ys = [base[0:100], base[200:300], base[400:500]]
+        plan.allreduce(xs, ys)
+        plan.sync()
+        with pytest.raises(DpdrError):
+            plan.set(N.OPT_FUSED_MODE, 5)
+        with pytest.raises(DpdrError):
+            plan.set(999, 1)
