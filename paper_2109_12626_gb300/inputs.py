@@ -120,7 +120,8 @@ def rank_values(kind: str, seed: int, rank: int, cols, device="cpu",
     """Values of one rank at the given columns, in the element layout the
     library uses: int32 / float32 as [n], 2x2 uint32 matrices as [n, 4]."""
     if kind == "int32":
-        return uniform_int32(seed, rank, cols, kw["lo"], kw["hi"], device)
+        return uniform_int32(seed, rank, cols, kw.get("lo", -1000),
+                             kw.get("hi", 1000), device)
     if kind == "float32":
         return normal_f32(seed, rank, cols, kw.get("sigma", 1.0), device)
     if kind == "mat2x2u32":
