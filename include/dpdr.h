@@ -181,6 +181,40 @@ int dpdr_allreduce_host(dpdr_plan_t plan, const void* const* x_host,
  * dpdr_last_error_message ("rank r round j step s"). */
 int dpdr_plan_sync(dpdr_plan_t plan, dpdr_stream_t stream);
 
+/* ------------------------------------------------------ allocation-free
+ * The paper has no counterpart to this entry point; it exists for callers
+ * that cannot allocate device memory on the call path: code whose device
+ * memory is owned by another allocator (a framework's caching pool, a fixed
+ * application-wide budget), or that must not call cudaMalloc while running
+ * because an allocation can fail mid-run or stall the whole device.  It
+ * needs no plan (dpdr_plan allocates) and calls no cudaMalloc, cudaFree or
+ * other allocating routine.
+ *
+ * It runs the same schedule kernel as dpdr_allreduce_schedule, with the same
+ * result, using a scratch array of DPDR_NOALLOC_SCRATCH_BYTES that is
+ * statically reserved in device memory on every GPU that loads the library
+ * and held until the process exits.  That array holds the rank-pointer and
+ * tree tables, the handshake counters, the error word and the dual roots'
+ * exchange slots (4 slots of one pipeline block each).  Limits: p <=
+ * DPDR_NOALLOC_MAX_RANKS, and the tables plus 4 slots of ceil(m/b) elements
+ * must fit the array; otherwise the call returns DPDR_ERR_INVALID saying
+ * which limit was hit (raise b to shrink the blocks).
+ *
+ * x and y are host arrays of p device pointers, as for dpdr_allreduce; the
+ * caller guarantees that no buffers overlap except y[i] == x[i] (this call
+ * does not check overlap).  b as for dpdr_plan (0 = block-count rule).
+ * The call is synchronous: it returns after stream has finished the
+ * kernel, with DPDR_ERR_TIMEOUT if one of its bounded waits expired.  The
+ * first call on each device looks up the array's device address (with that
+ * device current) and keeps it.  Every call shares the one array and
+ * re-initialises what must start at zero; calls that overlap on the GPU
+ * (from two host threads, or on two streams) race and must not be made. */
+#define DPDR_NOALLOC_SCRATCH_BYTES (8u << 20)
+#define DPDR_NOALLOC_MAX_RANKS 8192
+int dpdr_allreduce_schedule_noalloc(int p, int64_t m, dpdr_dtype dtype,
+                                    dpdr_op op, int b, const void* const* x,
+                                    void* const* y, dpdr_stream_t stream);
+
 /* ------------------------------------------------------------ errors */
 int dpdr_last_error(void);
 const char* dpdr_last_error_message(void);

@@ -40,6 +40,9 @@ SIGNATURES = {
     "dpdr_allreduce_schedule": (ctypes.c_int, [_P, _P, _P, _P]),
     "dpdr_allreduce_host": (ctypes.c_int, [_P, _P, _P, _P, _P, _P]),
     "dpdr_plan_sync": (ctypes.c_int, [_P, _P]),
+    "dpdr_allreduce_schedule_noalloc": (ctypes.c_int, [ctypes.c_int, ctypes.c_int64,
+                                                       ctypes.c_int, ctypes.c_int,
+                                                       ctypes.c_int, _P, _P, _P]),
     "dpdr_last_error": (ctypes.c_int, []),
     "dpdr_last_error_message": (ctypes.c_char_p, []),
     "dpdr_status_string": (ctypes.c_char_p, [ctypes.c_int]),

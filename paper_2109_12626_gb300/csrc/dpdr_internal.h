@@ -88,6 +88,9 @@ int block_count_rule(int p, int64_t m, double kappa);
 // errors (plan.cpp)
 int fail(int status, const std::string& msg);
 int cuda_fail(cudaError_t e, const char* what);
+// the same without building a std::string (no heap use)
+int fail_c(int status, const char* msg);
+int cuda_fail_c(cudaError_t e, const char* what);
 
 // rank-pointer upload (api.cpp)
 int stage_pointers(Plan* P, const void* const* x, const void* const* y,

@@ -22,6 +22,20 @@ int fail(int status, const std::string& msg)
     return status;
 }
 
+int fail_c(int status, const char* msg)
+{
+    g_last = status;
+    std::snprintf(g_msg, sizeof g_msg, "%s", msg);
+    return status;
+}
+
+int cuda_fail_c(cudaError_t e, const char* what)
+{
+    g_last = e == cudaErrorMemoryAllocation ? DPDR_ERR_OOM : DPDR_ERR_CUDA;
+    std::snprintf(g_msg, sizeof g_msg, "%s: %s", what, cudaGetErrorString(e));
+    return g_last;
+}
+
 int cuda_fail(cudaError_t e, const char* what)
 {
     std::string m = std::string(what) + ": " + cudaGetErrorString(e);

@@ -34,6 +34,7 @@
 // in time; an expired wait records {rank, round, step} in the plan's error
 // word, raises an abort flag that ends every other wait, and returns.
 #include <algorithm>
+#include <mutex>
 
 #include "dpdr_internal.h"
 #include "ops.cuh"
@@ -366,4 +367,227 @@ int schedule_launch(Plan* P, cudaStream_t s)
     return DPDR_OK;
 }
 
+
+// ------------------------------------------------------------- no-alloc
+// dpdr_allreduce_schedule_noalloc runs the schedule kernel above for
+// callers that cannot allocate device memory.  Everything the kernel needs
+// besides the caller's rank buffers -- the rank-pointer tables, the tree
+// tables, the CTA table, the handshake counters, the error word and the
+// dual roots' exchange slots -- lives in one file-scope device array that
+// exists on every GPU that loads this library until the process exits.
+// All calls share it, so two calls that overlap on the GPU race.
+constexpr size_t kNoAllocBytes = size_t(DPDR_NOALLOC_SCRATCH_BYTES);
+constexpr int kNoAllocMaxRanks = DPDR_NOALLOC_MAX_RANKS;
+constexpr int kNoAllocThreads = 128;
+constexpr int kNoAllocMaxDevices = 64;
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
+
+namespace {
+
+// Offsets inside the scratch array (bytes), for p ranks.
+struct NoAllocLayout {
+    size_t x, y, tables, ctrl, err, cta, ring, slot, end;
+};
+
+__host__ __device__ inline size_t na_align(size_t v) { return (v + 255) / 256 * 256; }
+
+inline NoAllocLayout noalloc_layout(int p, int64_t m, int b, size_t esize)
+{
+    NoAllocLayout L;
+    L.x = 0;
+    L.y = na_align(L.x + sizeof(void*) * size_t(p));
+    L.tables = na_align(L.y + sizeof(void*) * size_t(p));
+    L.ctrl = na_align(L.tables + sizeof(int) * 4 * size_t(p));
+    L.err = na_align(L.ctrl + sizeof(uint32_t) * (2 * size_t(p) + 1));
+    L.cta = na_align(L.err + sizeof(uint32_t) * 4);
+    L.ring = na_align(L.cta + sizeof(int) * (size_t(p) + 2));
+    const int64_t maxblk = (m + b - 1) / b + 4;
+    L.slot = na_align(size_t(maxblk) * esize + 16);
+    L.end = L.ring + 4 * L.slot;
+    return L;
+}
+
+// The complete-binary-tree split of a post-order interval of n ranks: the
+// size of the left (lower-ranked) subtree.
+__device__ __forceinline__ int left_size(int n)
+{
+    int H = 0;
+    while ((2 << H) <= n) H++;
+    const int half = 1 << (H - 1);
+    const int last = n - ((1 << H) - 1);
+    return (half - 1) + (last < half ? last : half);
+}
+
+// One thread per rank: parent, child0, child1 and depth by descending from
+// the root of the rank's tree; the first nctas+1 threads also write the CTA
+// table (R ranks per CTA, never straddling the trees).
+__global__ void noalloc_tables_kernel(int p, int R, int nctas, int* tables, int* cta_first)
+{
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    const int n0 = p / 2;
+    if (i < p) {
+        int lo = i < n0 ? 0 : n0, n = i < n0 ? n0 : p - n0;
+        int par = -1, d = 0;
+        while (true) {
+            const int root = lo + n - 1;
+            if (i == root) break;
+            const int L = left_size(n);
+            par = root;
+            d++;
+            if (i < lo + L) {
+                n = L;
+            } else {
+                lo += L;
+                n = n - 1 - L;
+            }
+        }
+        int c0 = -1, c1 = -1;
+        if (n > 1) {
+            const int L = left_size(n);
+            c0 = i - 1;
+            c1 = (n - 1 - L > 0) ? lo + L - 1 : -1;
+        }
+        tables[i] = par;
+        tables[p + i] = c0;
+        tables[2 * p + i] = c1;
+        tables[3 * p + i] = d;
+    }
+    if (i <= nctas) {
+        const int k0 = (n0 + R - 1) / R;
+        cta_first[i] = i < k0 ? i * R : (i < nctas ? n0 + (i - k0) * R : p);
+    }
+}
+
+std::mutex g_noalloc_mu;
+unsigned char* g_noalloc_ptr[kNoAllocMaxDevices];
+
+// Device address of the scratch array on the current device, looked up
+// once per device with that device current.
+int noalloc_scratch(unsigned char** out)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail_c(e, "no-alloc: cudaGetDevice");
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return fail_c(DPDR_ERR_INVALID, "no-alloc: device ordinal too large");
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void* ptr = nullptr;
+        e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+        if (e != cudaSuccess) return cuda_fail_c(e, "no-alloc: cudaGetSymbolAddress");
+        g_noalloc_ptr[dev] = static_cast<unsigned char*>(ptr);
+    }
+    *out = g_noalloc_ptr[dev];
+    return DPDR_OK;
+}
+
+}  // namespace
+
+int schedule_noalloc(int p, int64_t m, int dtype, int op, int b, const void* const* x,
+                     void* const* y, cudaStream_t s)
+{
+    if (p < 1 || m < 0) return fail_c(DPDR_ERR_INVALID, "no-alloc: need p >= 1 and m >= 0");
+    if (p > kNoAllocMaxRanks)
+        return fail_c(DPDR_ERR_INVALID, "no-alloc: p exceeds DPDR_NOALLOC_MAX_RANKS");
+    const bool sum_ok = (dtype == DPDR_INT32 || dtype == DPDR_FLOAT32) && op == DPDR_OP_SUM;
+    const bool mat_ok = dtype == DPDR_MAT2X2_U32 && op == DPDR_OP_MATMUL;
+    if (!sum_ok && !mat_ok) return fail_c(DPDR_ERR_INVALID, "no-alloc: unsupported (dtype, op)");
+    if (b < 0) return fail_c(DPDR_ERR_INVALID, "no-alloc: b < 0");
+    if (!x || !y) return fail_c(DPDR_ERR_INVALID, "no-alloc: x or y is NULL");
+    const size_t esize = dtype == DPDR_MAT2X2_U32 ? 16 : 4;
+    int vec = 1;
+    for (int i = 0; i < p; i++) {
+        const uintptr_t a = reinterpret_cast<uintptr_t>(x[i]), c = reinterpret_cast<uintptr_t>(y[i]);
+        if (!a || !c) return fail_c(DPDR_ERR_INVALID, "no-alloc: NULL rank buffer");
+        if ((a | c) & 3u) return fail_c(DPDR_ERR_INVALID, "no-alloc: rank buffer not 4-byte aligned");
+        if ((a | c) & 15u) vec = 0;
+    }
+    if (m == 0) return DPDR_OK;
+    const int64_t hi = m < (int64_t(1) << 30) ? m : (int64_t(1) << 30);
+    int bb = b == 0 ? block_count_rule(p, m, 0) : b;
+    bb = int(bb < 1 ? 1 : (bb > hi ? hi : bb));
+    const NoAllocLayout L = noalloc_layout(p, m, bb, esize);
+    if (L.end > kNoAllocBytes)
+        return fail_c(DPDR_ERR_INVALID,
+                      "no-alloc: pipeline block too large for DPDR_NOALLOC_SCRATCH_BYTES; "
+                      "use more blocks (larger b)");
+
+    unsigned char* base = nullptr;
+    int rc = noalloc_scratch(&base);
+    if (rc) return rc;
+    int dev = 0, sms = 0, occ = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e == cudaSuccess)
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kernel_for(dtype), kNoAllocThreads, 0);
+    if (e != cudaSuccess) return cuda_fail_c(e, "no-alloc: device query");
+    const int64_t kmax = int64_t(occ) * sms;
+    const int n0 = p / 2, n1 = p - n0;
+    int R = 1;
+    while (R < p && int64_t((n0 + R - 1) / R + (n1 + R - 1) / R) > kmax) R++;
+    const int nctas = (n0 + R - 1) / R + (n1 + R - 1) / R;
+
+    // rank pointers from the caller's host arrays, zeroed counters and
+    // error word, tree and CTA tables
+    e = cudaMemcpyAsync(base + L.x, x, sizeof(void*) * size_t(p), cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(base + L.y, y, sizeof(void*) * size_t(p), cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(base + L.ctrl, 0, L.cta - L.ctrl, s);
+    if (e != cudaSuccess) return cuda_fail_c(e, "no-alloc: set-up copies");
+    int* tables = reinterpret_cast<int*>(base + L.tables);
+    int* cta = reinterpret_cast<int*>(base + L.cta);
+    const int tb = 256, blocks = (p + 1 + tb - 1) / tb + 1;
+    noalloc_tables_kernel<<<blocks, tb, 0, s>>>(p, R, nctas, tables, cta);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail_c(e, "no-alloc: table kernel");
+
+    SchedArgs a;
+    a.x = reinterpret_cast<const char* const*>(base + L.x);
+    a.y = reinterpret_cast<char* const*>(base + L.y);
+    a.parent = tables;
+    a.child0 = tables + p;
+    a.child1 = tables + 2 * p;
+    a.depth = tables + 3 * p;
+    a.cta_first = cta;
+    uint32_t* ctrl = reinterpret_cast<uint32_t*>(base + L.ctrl);
+    a.up = ctrl;
+    a.down = ctrl + p;
+    a.abort_flag = ctrl + 2 * p;
+    a.err = reinterpret_cast<uint32_t*>(base + L.err);
+    a.ring = reinterpret_cast<char*>(base + L.ring);
+    a.ring_slot = int64_t(L.slot);
+    a.p = p;
+    a.b = bb;
+    a.r0 = p / 2 - 1;
+    a.r1 = p - 1;
+    a.m = m;
+    a.q = m / bb;
+    a.rem = m % bb;
+    a.wait_ns = 4000000000LL;
+    a.skip_rank = -1;
+    a.vec = vec;
+    void* args[] = {&a};
+    e = cudaLaunchCooperativeKernel(kernel_for(dtype), dim3(nctas), dim3(kNoAllocThreads), args, 0, s);
+    if (e == cudaErrorCooperativeLaunchTooLarge) {
+        cudaGetLastError();
+        return fail_c(DPDR_ERR_NOT_COOPERATIVE, "no-alloc: CTAs cannot be co-resident");
+    }
+    if (e != cudaSuccess) return cuda_fail_c(e, "no-alloc: schedule kernel launch");
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail_c(e, "no-alloc: stream synchronize");
+    uint32_t err[4] = {0, 0, 0, 0};
+    e = cudaMemcpy(err, base + L.err, sizeof err, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail_c(e, "no-alloc: error word read");
+    if (err[0] != 0) return fail_c(int(err[0]), "no-alloc: schedule wait expired");
+    return DPDR_OK;
+}
+
 }  // namespace dpdr
+
+extern "C" int dpdr_allreduce_schedule_noalloc(int p, int64_t m, dpdr_dtype dtype, dpdr_op op,
+                                               int b, const void* const* x, void* const* y,
+                                               dpdr_stream_t stream)
+{
+    return dpdr::schedule_noalloc(p, m, int(dtype), int(op), b, x, y,
+                                  reinterpret_cast<cudaStream_t>(stream));
+}
