@@ -115,7 +115,9 @@ int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
 
 /* Plan options (key, value):
  *   DPDR_OPT_FUSED_MODE       0 auto, 1 column-streaming, 2 shared-memory
- *                             tile (the two layouts of dpdr_allreduce)
+ *                             tile, 3 subtree split (the three layouts of
+ *                             dpdr_allreduce; 3 needs trees of depth >= 3
+ *                             and allocates m * esize bytes per subtree)
  *   DPDR_OPT_WAIT_LIMIT_NS    bound of every wait of the schedule kernel,
  *                             nanoseconds (default 4e9)
  *   DPDR_OPT_SKIP_RANK        fault injection for tests: this rank of the
@@ -139,7 +141,9 @@ int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
 /* Plan facts for tools and tests, int64 each, n of them:
  *   [0] p  [1] m  [2] b  [3] max depth  [4] fused mode that auto selects
  *   [5] schedule CTAs  [6] ranks per schedule CTA  [7] device scratch bytes
- *   [8] 1 if the last dpdr_allreduce ran the 16-byte vector path */
+ *   [8] 1 if the last dpdr_allreduce ran the 16-byte vector path
+ *   [9] split layout cut depth  [10] its subtrees  [11] ranks per store
+ *   group of its second kernel (0 when the split layout is not prepared) */
 int dpdr_plan_info(dpdr_plan_t plan, int64_t* info, int n);
 
 /* Releases the plan's device and host memory.  The caller must first make

@@ -174,11 +174,12 @@ class Plan:
         return out
 
     def info(self) -> dict:
-        v = np.zeros(9, np.int64)
-        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), 9),
+        v = np.zeros(12, np.int64)
+        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), 12),
                "dpdr_plan_info")
         keys = ("p", "m", "b", "max_depth", "auto_mode", "sched_ctas",
-                "sched_ranks_per_cta", "scratch_bytes", "vector_path")
+                "sched_ranks_per_cta", "scratch_bytes", "vector_path",
+                "split_depth", "split_subtrees", "split_group")
         return {k: int(x) for k, x in zip(keys, v)}
 
     def set(self, key: int, value: int) -> None:
@@ -205,6 +206,31 @@ class Plan:
                                          _ptr_array(xd), _ptr_array(yd),
                                          _stream(stream)), "dpdr_allreduce_host")
 
+    def bind(self, xs: Sequence, ys: Sequence) -> "Bound":
+        """Marshal the rank buffers once, for repeated calls on them."""
+        return Bound(self, xs, ys)
+
     def sync(self, stream=None) -> None:
         """Wait for the stream; raise DpdrError on a schedule-kernel timeout."""
         _check(lib().dpdr_plan_sync(self._h, _stream(stream)), "dpdr_plan_sync")
+
+
+class Bound:
+    """A plan with its rank-pointer arrays marshalled once (repeated calls
+    on the same buffers cost one C call each)."""
+
+    def __init__(self, plan: Plan, xs: Sequence, ys: Sequence):
+        assert len(xs) == plan.p and len(ys) == plan.p
+        self.plan = plan
+        self._keep = (list(xs), list(ys))
+        self.X = _ptr_array(xs)
+        self.Y = _ptr_array(ys)
+
+    def allreduce(self, stream=None) -> None:
+        _check(lib().dpdr_allreduce(self.plan._h, self.X, self.Y, _stream(stream)),
+               "dpdr_allreduce")
+
+    def allreduce_schedule(self, stream=None) -> None:
+        _check(lib().dpdr_allreduce_schedule(self.plan._h, self.X, self.Y,
+                                             _stream(stream)),
+               "dpdr_allreduce_schedule")

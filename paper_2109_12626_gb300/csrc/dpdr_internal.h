@@ -75,6 +75,20 @@ struct Plan {
     cudaEvent_t staged = nullptr;
     bool staged_pending = false;     // d_x / d_y hold last_x / last_y
 
+    // dynamic shared memory already granted to the fused kernels of this
+    // plan's element type (stream, tile), so launches skip the attribute call
+    int smem_attr[3] = {48 * 1024, 48 * 1024, 48 * 1024};
+
+    // split layout of the fused kernel (fused.cu): subtrees at depth split_s
+    bool split_ready = false;
+    int split_s = 0, split_nseg = 0, split_nitems = 0, split_group = 1;
+    char* d_split = nullptr;         // own allocation: seg, items, subtree rows
+    size_t d_split_bytes = 0;
+    int2* d_seg = nullptr;
+    int2* d_items = nullptr;
+    char* d_part = nullptr;
+    int64_t part_stride = 0;
+
     // facts
     int last_vector_path = 0;
     int sched_ctas = 0, sched_ranks_per_cta = 0;
@@ -99,6 +113,7 @@ int stage_pointers(Plan* P, const void* const* x, const void* const* y,
 // launchers
 int fused_launch(Plan* P, cudaStream_t s);      // fused.cu
 int fused_auto_mode(const Plan* P);             // fused.cu
+int fused_split_prepare(Plan* P, bool force);   // fused.cu
 int schedule_launch(Plan* P, cudaStream_t s);   // schedule.cu
 int schedule_configure(Plan* P);                // schedule.cu
 

@@ -47,6 +47,13 @@ struct FusedArgs {
     int64_t scalar_base;    // element index of the first single element
     int lg_wu;              // tile: log2 of vector units per row
     int64_t vec_tiles;      // tile: number of vector tiles
+    // split layout
+    const int2* seg;        // [nseg] (first rank, root rank) of each subtree
+    const int2* items;      // [nitems] top fold: (source, tape byte | kind << 8)
+    int nitems;
+    char* part;             // [nseg] rows of subtree values
+    int64_t part_stride;    // bytes per row
+    int group;              // ranks stored by one CTA row of the finish kernel
 };
 
 template <class Op>
@@ -61,6 +68,15 @@ struct VecUnit {
         st_stream(row + u * 16, v);
     }
     __device__ __forceinline__ static T op(const T& a, const T& b) { return Op::vec(a, b); }
+    // data read again soon (subtree values, top-of-tree inputs): keep in L2
+    __device__ __forceinline__ static T ld_keep(const char* row, int64_t u)
+    {
+        return ld_l2(row + u * 16);
+    }
+    __device__ __forceinline__ static void st_keep(char* row, int64_t u, const T& v)
+    {
+        st_l2(row + u * 16, v);
+    }
 };
 
 template <class Op>
@@ -75,6 +91,14 @@ struct OneUnit {
         st_one_stream<Op>(row + e * Op::kEsize, v);
     }
     __device__ __forceinline__ static T op(const T& a, const T& b) { return comb<Op>(a, b); }
+    __device__ __forceinline__ static T ld_keep(const char* row, int64_t e)
+    {
+        return ld_one_l2<Op>(row + e * Op::kEsize);
+    }
+    __device__ __forceinline__ static void st_keep(char* row, int64_t e, const T& v)
+    {
+        st_one_l2<Op>(row + e * Op::kEsize, v);
+    }
 };
 
 __device__ __forceinline__ const char* rank_ptr(const char* const* t, int i)
@@ -87,6 +111,22 @@ __device__ __forceinline__ char* rank_ptr_w(char* const* t, int i)
 }
 
 // ---------------------------------------------------------------- streaming
+// One step of the running post-order fold: v is rank i's own value x_i (or,
+// in the split layout, a whole subtree's value with no children left); acc
+// holds the value of rank i-1, which is child_0 whenever i has a child; a
+// child_1 value waits in slot[depth+1]; a node that is a child_1 (or the
+// lower root) parks its value in slot[depth].
+template <class U>
+__device__ __forceinline__ void fold_step(unsigned t, typename U::T v, typename U::T& acc,
+                                          typename U::T* slot, int stride)
+{
+    const unsigned c = t & 3u, d = (t >> 3) & 31u;
+    if (c >= 1) v = U::op(acc, v);                     // v(c0) (.) x_i
+    if (c == 2) v = U::op(slot[(d + 1) * stride], v);  // v(c1) (.) (..)
+    if (t & kTapeKeep) slot[d * stride] = v;
+    acc = v;
+}
+
 template <class U>
 __device__ __forceinline__ void stream_column(const FusedArgs& a, int64_t u,
                                               typename U::T* slot, int stride)
@@ -106,17 +146,8 @@ __device__ __forceinline__ void stream_column(const FusedArgs& a, int64_t u,
         const unsigned long long tp =
             __ldg(reinterpret_cast<const unsigned long long*>(a.tape + i0));
 #pragma unroll
-        for (int k = 0; k < kStreamAhead; k++) {
-            if (i0 + k < p) {
-                const unsigned t = unsigned(tp >> (8 * k)) & 0xffu;
-                const unsigned c = t & 3u, d = t >> 3;
-                T v = cur[k];
-                if (c >= 1) v = U::op(acc, v);                     // v(c0) (.) x_i
-                if (c == 2) v = U::op(slot[(d + 1) * stride], v);  // v(c1) (.) (..)
-                if (t & kTapeKeep) slot[d * stride] = v;
-                acc = v;
-            }
-        }
+        for (int k = 0; k < kStreamAhead; k++)
+            if (i0 + k < p) fold_step<U>(unsigned(tp >> (8 * k)) & 0xffu, cur[k], acc, slot, stride);
 #pragma unroll
         for (int k = 0; k < kStreamAhead; k++) cur[k] = nxt[k];
     }
@@ -136,6 +167,103 @@ fused_stream_kernel(FusedArgs a)
     } else if (u < a.nvec + a.nscalar) {
         auto* slot = reinterpret_cast<Elem<Op>*>(smem) + threadIdx.x;
         stream_column<OneUnit<Op>>(a, a.scalar_base + (u - a.nvec), slot, blockDim.x);
+    }
+}
+
+// -------------------------------------------------------------------- split
+// For m too small to give every SM enough columns but p large: the rank axis
+// is cut at a tree depth s.  Kernel 1 folds each depth-s subtree (a
+// contiguous post-order interval) for its columns, in parallel over
+// (subtree, column) and writes the subtree value to a scratch row.  Kernel 2
+// folds the nodes above depth s, reading each subtree as one finished child,
+// forms v(r0) (.) v(r1), and stores it to one group of ranks per CTA row.
+// The bracketing is unchanged: each subtree value is exactly its node value.
+template <class U>
+__device__ __forceinline__ void split_reduce_column(const FusedArgs& a, int g, int64_t u,
+                                                    typename U::T* slot, int stride)
+{
+    using T = typename U::T;
+    const int2 sg = __ldg(a.seg + g);
+    const int lo = sg.x, hi = sg.y;  // inclusive; lo is a leaf
+    T cur[kStreamAhead], nxt[kStreamAhead];
+#pragma unroll
+    for (int k = 0; k < kStreamAhead; k++)
+        if (lo + k <= hi) cur[k] = U::ld(rank_ptr(a.x, lo + k), u);
+    T acc = cur[0];
+    for (int i0 = lo; i0 <= hi; i0 += kStreamAhead) {
+#pragma unroll
+        for (int k = 0; k < kStreamAhead; k++)
+            if (i0 + kStreamAhead + k <= hi)
+                nxt[k] = U::ld(rank_ptr(a.x, i0 + kStreamAhead + k), u);
+#pragma unroll
+        for (int k = 0; k < kStreamAhead; k++)
+            if (i0 + k <= hi) fold_step<U>(__ldg(a.tape + i0 + k), cur[k], acc, slot, stride);
+#pragma unroll
+        for (int k = 0; k < kStreamAhead; k++) cur[k] = nxt[k];
+    }
+    U::st_keep(a.part + int64_t(g) * a.part_stride, u, acc);
+}
+
+template <class U>
+__device__ __forceinline__ void split_finish_column(const FusedArgs& a, int r, int64_t u,
+                                                    typename U::T* slot, int stride)
+{
+    using T = typename U::T;
+    const int n = a.nitems;
+    T cur[kStreamAhead], nxt[kStreamAhead];
+    auto load = [&](int k) -> T {
+        const int2 it = __ldg(a.items + k);
+        return (it.y >> 8) ? U::ld_keep(a.part + int64_t(it.x) * a.part_stride, u)
+                           : U::ld_keep(rank_ptr(a.x, it.x), u);
+    };
+#pragma unroll
+    for (int k = 0; k < kStreamAhead; k++)
+        if (k < n) cur[k] = load(k);
+    T acc = cur[0];
+    for (int k0 = 0; k0 < n; k0 += kStreamAhead) {
+#pragma unroll
+        for (int k = 0; k < kStreamAhead; k++)
+            if (k0 + kStreamAhead + k < n) nxt[k] = load(k0 + kStreamAhead + k);
+#pragma unroll
+        for (int k = 0; k < kStreamAhead; k++)
+            if (k0 + k < n)
+                fold_step<U>(unsigned(__ldg(&a.items[k0 + k].y)) & 0xffu, cur[k], acc, slot, stride);
+#pragma unroll
+        for (int k = 0; k < kStreamAhead; k++) cur[k] = nxt[k];
+    }
+    const T y = (a.p >= 2) ? U::op(slot[0], acc) : acc;
+    const int i1 = min(a.p, (r + 1) * a.group);
+#pragma unroll 4
+    for (int i = r * a.group; i < i1; i++) U::st(rank_ptr_w(a.y, i), u, y);
+}
+
+template <class Op>
+__global__ void __launch_bounds__(kStreamThreads, 3)
+fused_split_reduce_kernel(FusedArgs a)
+{
+    extern __shared__ uint4 smem[];
+    const int64_t u = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (u < a.nvec) {
+        split_reduce_column<VecUnit<Op>>(a, blockIdx.y, u, smem + threadIdx.x, blockDim.x);
+    } else if (u < a.nvec + a.nscalar) {
+        auto* slot = reinterpret_cast<Elem<Op>*>(smem) + threadIdx.x;
+        split_reduce_column<OneUnit<Op>>(a, blockIdx.y, a.scalar_base + (u - a.nvec), slot,
+                                         blockDim.x);
+    }
+}
+
+template <class Op>
+__global__ void __launch_bounds__(kStreamThreads, 3)
+fused_split_finish_kernel(FusedArgs a)
+{
+    extern __shared__ uint4 smem[];
+    const int64_t u = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (u < a.nvec) {
+        split_finish_column<VecUnit<Op>>(a, blockIdx.y, u, smem + threadIdx.x, blockDim.x);
+    } else if (u < a.nvec + a.nscalar) {
+        auto* slot = reinterpret_cast<Elem<Op>*>(smem) + threadIdx.x;
+        split_finish_column<OneUnit<Op>>(a, blockIdx.y, a.scalar_base + (u - a.nvec), slot,
+                                         blockDim.x);
     }
 }
 
@@ -226,21 +354,47 @@ int launch(Plan* P, FusedArgs a, int mode, cudaStream_t s)
         const int64_t blocks = (units + kStreamThreads - 1) / kStreamThreads;
         const size_t smem = size_t(P->max_depth + 1) * kStreamThreads * sizeof(uint4);
         if (blocks > 0x7fffffff) return fail(DPDR_ERR_INVALID, "m too large");
-        cudaError_t e = cudaFuncSetAttribute(fused_stream_kernel<Op>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             int(smem));
-        if (e != cudaSuccess) return cuda_fail(e, "fused stream attribute");
+        if (int(smem) > P->smem_attr[0]) {
+            cudaError_t e = cudaFuncSetAttribute(fused_stream_kernel<Op>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 int(smem));
+            if (e != cudaSuccess) return cuda_fail(e, "fused stream attribute");
+            P->smem_attr[0] = int(smem);
+        }
         fused_stream_kernel<Op><<<unsigned(blocks), kStreamThreads, smem, s>>>(a);
+    } else if (mode == 3) {
+        const int64_t units = a.nvec + a.nscalar;
+        const int64_t blocks = (units + kStreamThreads - 1) / kStreamThreads;
+        const size_t smem = size_t(P->max_depth + 1) * kStreamThreads * sizeof(uint4);
+        if (blocks > 0x7fffffff) return fail(DPDR_ERR_INVALID, "m too large");
+        if (int(smem) > P->smem_attr[2]) {
+            cudaError_t e = cudaFuncSetAttribute(fused_split_reduce_kernel<Op>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 int(smem));
+            if (e == cudaSuccess)
+                e = cudaFuncSetAttribute(fused_split_finish_kernel<Op>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+            if (e != cudaSuccess) return cuda_fail(e, "fused split attribute");
+            P->smem_attr[2] = int(smem);
+        }
+        const int groups = (P->p + a.group - 1) / a.group;
+        fused_split_reduce_kernel<Op>
+            <<<dim3(unsigned(blocks), unsigned(P->split_nseg)), kStreamThreads, smem, s>>>(a);
+        fused_split_finish_kernel<Op>
+            <<<dim3(unsigned(blocks), unsigned(groups)), kStreamThreads, smem, s>>>(a);
     } else {
         const size_t smem = size_t(P->p + 1) * (size_t(16) << a.lg_wu);
         const int64_t lg_s = a.lg_wu + (Op::kEsize == 4 ? 2 : 0);
         const int64_t scal_tiles = (a.nscalar + (int64_t(1) << lg_s) - 1) >> lg_s;
         const int64_t blocks = a.vec_tiles + scal_tiles;
         if (blocks > 0x7fffffff) return fail(DPDR_ERR_INVALID, "m too large");
-        cudaError_t e = cudaFuncSetAttribute(fused_tile_kernel<Op>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             int(smem));
-        if (e != cudaSuccess) return cuda_fail(e, "fused tile attribute");
+        if (int(smem) > P->smem_attr[1]) {
+            cudaError_t e = cudaFuncSetAttribute(fused_tile_kernel<Op>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 int(smem));
+            if (e != cudaSuccess) return cuda_fail(e, "fused tile attribute");
+            P->smem_attr[1] = int(smem);
+        }
         fused_tile_kernel<Op><<<unsigned(blocks), kTileThreads, smem, s>>>(a);
     }
     cudaError_t e = cudaGetLastError();
@@ -260,12 +414,71 @@ int tile_lg_wu(const Plan* P)
 
 }  // namespace
 
+// Threads the streaming layouts want in flight to cover HBM latency.
+static int64_t stream_target(const Plan* P) { return int64_t(P->num_sms) * 1024; }
+
 int fused_auto_mode(const Plan* P)
 {
-    if (tile_lg_wu(P) < 0) return 1;
     const int64_t units = P->m * int64_t(P->esize) / 16;
     // column streaming needs enough independent columns to fill every SM
-    return units >= int64_t(P->num_sms) * 1024 ? 1 : 2;
+    if (units >= stream_target(P)) return 1;
+    if (P->split_nseg > 0 && units * P->split_nseg >= int64_t(P->num_sms) * 256) return 3;
+    return tile_lg_wu(P) < 0 ? (P->split_nseg > 0 ? 3 : 1) : 2;
+}
+
+// Split layout: cut depth s, subtree table, top-of-tree item list, rank
+// groups of the finish kernel, and the scratch rows of subtree values.
+int fused_split_prepare(Plan* P, bool force)
+{
+    if (P->split_ready) return DPDR_OK;
+    const int p = P->p;
+    if (P->max_depth < 3) return DPDR_OK;  // nothing worth splitting
+    const int64_t units = std::max<int64_t>(1, P->m * int64_t(P->esize) / 16);
+    const int64_t target = stream_target(P);
+    if (!force && units >= target) return DPDR_OK;  // auto never picks it
+    int s = 1;
+    for (; s < P->max_depth - 2; s++) {
+        int64_t n = 0;
+        for (int i = 0; i < p; i++) n += P->depth[i] == s;
+        if (n * units >= target) break;
+    }
+    std::vector<int2> seg, items;
+    for (int i = 0; i < p; i++) {
+        if (P->depth[i] > s) continue;
+        if (P->depth[i] == s) {
+            int lo = i;  // leftmost leaf of the subtree
+            while (P->child0[lo] >= 0) lo = P->child1[lo] >= 0 ? P->child1[lo] : P->child0[lo];
+            items.push_back(make_int2(int(seg.size()), int(P->tape[i] & ~3u) | (1 << 8)));
+            seg.push_back(make_int2(lo, i));
+        } else {
+            items.push_back(make_int2(i, int(P->tape[i])));
+        }
+    }
+    int64_t groups = std::min<int64_t>(p, std::max<int64_t>(1, (target + units - 1) / units));
+    P->split_group = int((p + groups - 1) / groups);
+    P->split_s = s;
+    P->split_nseg = int(seg.size());
+    P->split_nitems = int(items.size());
+    P->part_stride = int64_t((size_t(P->m) * P->esize + 255) / 256 * 256);
+    const size_t o_items = (sizeof(int2) * seg.size() + 255) / 256 * 256;
+    const size_t o_part = o_items + (sizeof(int2) * items.size() + 255) / 256 * 256;
+    const size_t bytes = o_part + size_t(P->part_stride) * seg.size();
+    cudaError_t e = cudaMalloc(&P->d_split, bytes);
+    if (e != cudaSuccess) {
+        P->split_nseg = 0;
+        return cuda_fail(e, "split layout: cudaMalloc");
+    }
+    P->d_split_bytes = bytes;
+    P->d_seg = reinterpret_cast<int2*>(P->d_split);
+    P->d_items = reinterpret_cast<int2*>(P->d_split + o_items);
+    P->d_part = P->d_split + o_part;
+    e = cudaMemcpy(P->d_seg, seg.data(), sizeof(int2) * seg.size(), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess)
+        e = cudaMemcpy(P->d_items, items.data(), sizeof(int2) * items.size(),
+                       cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "split layout: upload");
+    P->split_ready = true;
+    return DPDR_OK;
 }
 
 int fused_launch(Plan* P, cudaStream_t s)
@@ -274,6 +487,7 @@ int fused_launch(Plan* P, cudaStream_t s)
     int mode = P->fused_mode ? P->fused_mode : fused_auto_mode(P);
     const int lg = tile_lg_wu(P);
     if (mode == 2 && lg < 0) return fail(DPDR_ERR_INVALID, "tile mode: p too large");
+    if (mode == 3 && !P->split_ready) return fail(DPDR_ERR_INVALID, "split mode: p too small");
 
     FusedArgs a;
     a.x = P->d_x;
@@ -292,6 +506,12 @@ int fused_launch(Plan* P, cudaStream_t s)
     a.nscalar = P->m - a.scalar_base;
     a.lg_wu = lg < 0 ? 0 : lg;
     a.vec_tiles = (a.nvec + (int64_t(1) << a.lg_wu) - 1) >> a.lg_wu;
+    a.seg = P->d_seg;
+    a.items = P->d_items;
+    a.nitems = P->split_nitems;
+    a.part = P->d_part;
+    a.part_stride = P->part_stride;
+    a.group = P->split_group;
 
     switch (P->dtype) {
     case DPDR_INT32: return launch<SumI32>(P, a, mode, s);

@@ -209,6 +209,7 @@ static void free_plan(Plan* P)
 {
     if (!P) return;
     if (P->staged) cudaEventDestroy(P->staged);
+    if (P->d_split) cudaFree(P->d_split);
     if (P->h_ptrs) cudaFreeHost(P->h_ptrs);
     if (P->dmem) cudaFree(P->dmem);
     delete P;
@@ -326,7 +327,8 @@ extern "C" dpdr_plan_t dpdr_plan(int p, int64_t m, dpdr_dtype dtype,
         free_plan(P);
         return nullptr;
     }
-    if (allocate(P) != DPDR_OK || schedule_configure(P) != DPDR_OK) {
+    if (allocate(P) != DPDR_OK || schedule_configure(P) != DPDR_OK ||
+        fused_split_prepare(P, false) != DPDR_OK) {
         free_plan(P);
         return nullptr;
     }
@@ -355,7 +357,12 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
     if (!P) return fail(DPDR_ERR_INVALID, "dpdr_plan_set: NULL plan");
     switch (key) {
     case DPDR_OPT_FUSED_MODE:
-        if (v < 0 || v > 2) return fail(DPDR_ERR_INVALID, "fused mode: 0, 1 or 2");
+        if (v < 0 || v > 3) return fail(DPDR_ERR_INVALID, "fused mode: 0, 1, 2 or 3");
+        if (v == 3) {
+            int rc = fused_split_prepare(P, true);
+            if (rc) return rc;
+            if (!P->split_ready) return fail(DPDR_ERR_INVALID, "split mode needs trees of depth >= 3");
+        }
         P->fused_mode = int(v);
         return DPDR_OK;
     case DPDR_OPT_WAIT_LIMIT_NS:
@@ -399,7 +406,8 @@ extern "C" int dpdr_plan_info(dpdr_plan_t h, int64_t* info, int n)
     if (!P || !info) return fail(DPDR_ERR_INVALID, "dpdr_plan_info: NULL");
     const int64_t v[] = {P->p, P->m, P->b, P->max_depth, fused_auto_mode(P),
                          P->sched_ctas, P->sched_ranks_per_cta,
-                         int64_t(P->dmem_bytes), P->last_vector_path};
+                         int64_t(P->dmem_bytes + P->d_split_bytes), P->last_vector_path,
+                         P->split_s, P->split_nseg, P->split_group};
     const int k = int(sizeof v / sizeof v[0]);
     for (int i = 0; i < n; i++) info[i] = i < k ? v[i] : 0;
     return DPDR_OK;

@@ -56,7 +56,7 @@ def _check_all(ys, want, guards=None):
 
 
 @pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
-@pytest.mark.parametrize("mode", [1, 2], ids=["stream", "tile"])
+@pytest.mark.parametrize("mode", [1, 2, 3], ids=["stream", "tile", "split"])
 def test_fused_matches_oracle(pkg, orc, case, mode):
     _, kind, seed, p, m, kw, _ = case
     dev = torch.device("cuda:0")
@@ -65,6 +65,8 @@ def test_fused_matches_oracle(pkg, orc, case, mode):
     xs, _ = to_device(x, kind, dev)
     ys, _ = empty_like_ranks(xs)
     with pkg.Plan(p, m, kind, 4) as plan:
+        if mode == 3 and plan.info()["max_depth"] < 3:
+            pytest.skip("split layout needs trees of depth >= 3")
         plan.set(pkg.OPT_FUSED_MODE, mode)
         plan.allreduce(xs, ys)
         plan.sync()
@@ -91,27 +93,37 @@ def test_schedule_matches_oracle(pkg, orc, case):
         assert np.array_equal(bits(xs[i]), expect_bits(x[i]))
 
 
+FUSED_RUNS = {"fused_stream": 1, "fused_tile": 2, "fused_split": 3}
+RUNS = list(FUSED_RUNS) + ["schedule"]
+
+
+def _run(pkg, plan, run, xs, ys):
+    if run == "schedule":
+        plan.allreduce_schedule(xs, ys)
+    else:
+        if FUSED_RUNS[run] == 3 and plan.info()["max_depth"] < 3:
+            pytest.skip("split layout needs trees of depth >= 3")
+        plan.set(pkg.OPT_FUSED_MODE, FUSED_RUNS[run])
+        plan.allreduce(xs, ys)
+
+
 @pytest.mark.parametrize("kind,p,m", [("int32", 7, 1000), ("float32", 1152, 4099),
                                       ("mat2x2u32", 36, 999), ("float32", 2, 5)])
-@pytest.mark.parametrize("run", ["fused_stream", "fused_tile", "schedule"])
+@pytest.mark.parametrize("run", RUNS)
 def test_in_place(pkg, orc, kind, p, m, run):
     """y[i] == x[i]: Algorithm 1 works in place (Y <- x_i, y ends in Y)."""
     x = host_inputs(kind, 11, p, m)
     want = _want(orc, x, kind)
     xs, _ = to_device(x, kind, torch.device("cuda:0"))
     with pkg.Plan(p, m, kind, 3) as plan:
-        if run == "schedule":
-            plan.allreduce_schedule(xs, xs)
-        else:
-            plan.set(pkg.OPT_FUSED_MODE, 1 if run == "fused_stream" else 2)
-            plan.allreduce(xs, xs)
+        _run(pkg, plan, run, xs, xs)
         plan.sync()
     _check_all(xs, want)
 
 
 @pytest.mark.parametrize("kind,p,m", [("int32", 7, 1001), ("float32", 1152, 133),
                                       ("mat2x2u32", 36, 257), ("float32", 32, 9999)])
-@pytest.mark.parametrize("run", ["fused_stream", "fused_tile", "schedule"])
+@pytest.mark.parametrize("run", RUNS)
 def test_four_byte_aligned_buffers(pkg, orc, kind, p, m, run):
     """Buffers only 4-byte aligned take the single-element paths."""
     x = host_inputs(kind, 12, p, m)
@@ -120,17 +132,13 @@ def test_four_byte_aligned_buffers(pkg, orc, kind, p, m, run):
     xs, keep_x = to_device(x, kind, dev, pad_front=1)
     ys, keep_y = empty_like_ranks(xs, pad_front=3)
     with pkg.Plan(p, m, kind, 4) as plan:
-        if run == "schedule":
-            plan.allreduce_schedule(xs, ys)
-        else:
-            plan.set(pkg.OPT_FUSED_MODE, 1 if run == "fused_stream" else 2)
-            plan.allreduce(xs, ys)
+        _run(pkg, plan, run, xs, ys)
         plan.sync()
         assert plan.info()["vector_path"] == 0
     _check_all(ys, want)
 
 
-@pytest.mark.parametrize("run", ["fused_stream", "fused_tile", "schedule"])
+@pytest.mark.parametrize("run", RUNS)
 def test_guard_words_untouched(pkg, orc, run):
     """No kernel writes past the m elements of an output."""
     kind, p, m = "float32", 36, 4097
@@ -141,11 +149,7 @@ def test_guard_words_untouched(pkg, orc, run):
     bases = [torch.full((m + 64,), 7.25, device=dev) for _ in range(p)]
     ys = [bb[:m] for bb in bases]
     with pkg.Plan(p, m, kind, 5) as plan:
-        if run == "schedule":
-            plan.allreduce_schedule(xs, ys)
-        else:
-            plan.set(pkg.OPT_FUSED_MODE, 1 if run == "fused_stream" else 2)
-            plan.allreduce(xs, ys)
+        _run(pkg, plan, run, xs, ys)
         plan.sync()
     _check_all(ys, want)
     for bb in bases:
