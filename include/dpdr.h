@@ -142,7 +142,8 @@ int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
  *   [0] p  [1] m  [2] b  [3] max depth  [4] fused mode that auto selects
  *   [5] schedule CTAs  [6] ranks per schedule CTA  [7] device scratch bytes
  *   [8] 1 if the last dpdr_allreduce ran the 16-byte vector path
- *   [9] split layout cut depth  [10] its subtrees  [11] ranks per store
+ *   [9] split layout cut depth  [10] its scratch rows (subtrees plus nodes
+ *   above the cut)  [11] ranks per store
  *   group of its second kernel (0 when the split layout is not prepared) */
 int dpdr_plan_info(dpdr_plan_t plan, int64_t* info, int n);
 

@@ -174,17 +174,24 @@ fused_stream_kernel(FusedArgs a)
 // For m too small to give every SM enough columns but p large: the rank axis
 // is cut at a tree depth s.  Kernel 1 folds each depth-s subtree (a
 // contiguous post-order interval) for its columns, in parallel over
-// (subtree, column) and writes the subtree value to a scratch row.  Kernel 2
-// folds the nodes above depth s, reading each subtree as one finished child,
-// forms v(r0) (.) v(r1), and stores it to one group of ranks per CTA row.
-// The bracketing is unchanged: each subtree value is exactly its node value.
+// (subtree, column), and writes the subtree value to a scratch row; it also
+// copies the inputs of the nodes above depth s into scratch rows.  Kernel 2
+// folds the nodes above depth s from those rows, each subtree entering as
+// one finished child, forms v(r0) (.) v(r1), and stores it to one group of
+// ranks per CTA row.  The bracketing is unchanged: each subtree value is
+// exactly its node value.
 template <class U>
 __device__ __forceinline__ void split_reduce_column(const FusedArgs& a, int g, int64_t u,
                                                     typename U::T* slot, int stride)
 {
     using T = typename U::T;
     const int2 sg = __ldg(a.seg + g);
-    const int lo = sg.x, hi = sg.y;  // inclusive; lo is a leaf
+    const int lo = sg.x, hi = sg.y;  // inclusive; lo is a leaf unless lo == hi
+    char* row = a.part + int64_t(g) * a.part_stride;
+    if (lo == hi) {  // a one-leaf subtree, or a node above the cut: its input
+        U::st_keep(row, u, U::ld(rank_ptr(a.x, lo), u));
+        return;
+    }
     T cur[kStreamAhead], nxt[kStreamAhead];
 #pragma unroll
     for (int k = 0; k < kStreamAhead; k++)
@@ -201,7 +208,7 @@ __device__ __forceinline__ void split_reduce_column(const FusedArgs& a, int g, i
 #pragma unroll
         for (int k = 0; k < kStreamAhead; k++) cur[k] = nxt[k];
     }
-    U::st_keep(a.part + int64_t(g) * a.part_stride, u, acc);
+    U::st_keep(row, u, acc);
 }
 
 template <class U>
@@ -211,10 +218,11 @@ __device__ __forceinline__ void split_finish_column(const FusedArgs& a, int r, i
     using T = typename U::T;
     const int n = a.nitems;
     T cur[kStreamAhead], nxt[kStreamAhead];
+    // every item is a scratch row: a subtree value or a copied input, so
+    // this kernel never reads an input that another CTA may be overwriting
+    // with the result (in-place use)
     auto load = [&](int k) -> T {
-        const int2 it = __ldg(a.items + k);
-        return (it.y >> 8) ? U::ld_keep(a.part + int64_t(it.x) * a.part_stride, u)
-                           : U::ld_keep(rank_ptr(a.x, it.x), u);
+        return U::ld_keep(a.part + int64_t(__ldg(&a.items[k].x)) * a.part_stride, u);
     };
 #pragma unroll
     for (int k = 0; k < kStreamAhead; k++)
@@ -442,17 +450,17 @@ int fused_split_prepare(Plan* P, bool force)
         for (int i = 0; i < p; i++) n += P->depth[i] == s;
         if (n * units >= target) break;
     }
+    // scratch rows: one per depth-s subtree (first rank, root), one per node
+    // above the cut (its own input, first = root); items in post-order
     std::vector<int2> seg, items;
     for (int i = 0; i < p; i++) {
         if (P->depth[i] > s) continue;
-        if (P->depth[i] == s) {
-            int lo = i;  // leftmost leaf of the subtree
+        int lo = i;
+        if (P->depth[i] == s)  // leftmost leaf of the subtree
             while (P->child0[lo] >= 0) lo = P->child1[lo] >= 0 ? P->child1[lo] : P->child0[lo];
-            items.push_back(make_int2(int(seg.size()), int(P->tape[i] & ~3u) | (1 << 8)));
-            seg.push_back(make_int2(lo, i));
-        } else {
-            items.push_back(make_int2(i, int(P->tape[i])));
-        }
+        const unsigned t = P->depth[i] == s ? (P->tape[i] & ~3u) : P->tape[i];
+        items.push_back(make_int2(int(seg.size()), int(t)));
+        seg.push_back(make_int2(lo, i));
     }
     int64_t groups = std::min<int64_t>(p, std::max<int64_t>(1, (target + units - 1) / units));
     P->split_group = int((p + groups - 1) / groups);
