@@ -116,8 +116,8 @@ int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
 /* Plan options (key, value):
  *   DPDR_OPT_FUSED_MODE       0 auto, 1 column-streaming, 2 shared-memory
  *                             tile, 3 subtree split (the three layouts of
- *                             dpdr_allreduce; 3 needs trees of depth >= 3
- *                             and allocates m * esize bytes per subtree)
+ *                             dpdr_allreduce; 3 needs p >= 2 and keeps
+ *                             m * esize bytes of scratch per subtree)
  *   DPDR_OPT_WAIT_LIMIT_NS    bound of every wait of the schedule kernel,
  *                             nanoseconds (default 4e9)
  *   DPDR_OPT_SKIP_RANK        fault injection for tests: this rank of the
@@ -127,14 +127,17 @@ int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
  *                             (64..256, multiple of 32; default 128)
  *   DPDR_OPT_SCHED_RANKS_PER_CTA  virtual ranks per CTA (0 = fewest that
  *                             fit co-resident)
- *   DPDR_OPT_BLOCKS           change b (same rules as dpdr_plan's b) */
+ *   DPDR_OPT_BLOCKS           change b (same rules as dpdr_plan's b)
+ *   DPDR_OPT_SPLIT_DEPTH      tree depth at which the split layout cuts
+ *                             the ranks into subtrees (-1 = automatic) */
 enum {
     DPDR_OPT_FUSED_MODE = 1,
     DPDR_OPT_WAIT_LIMIT_NS = 2,
     DPDR_OPT_SKIP_RANK = 3,
     DPDR_OPT_SCHED_THREADS = 4,
     DPDR_OPT_SCHED_RANKS_PER_CTA = 5,
-    DPDR_OPT_BLOCKS = 6
+    DPDR_OPT_BLOCKS = 6,
+    DPDR_OPT_SPLIT_DEPTH = 7
 };
 int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
 

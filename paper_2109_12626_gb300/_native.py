@@ -17,7 +17,7 @@ DPDR_OP_SUM, DPDR_OP_MATMUL = 0, 1
 (DPDR_OK, DPDR_ERR_INVALID, DPDR_ERR_CUDA, DPDR_ERR_TIMEOUT,
  DPDR_ERR_NOT_COOPERATIVE, DPDR_ERR_OOM) = range(6)
 (OPT_FUSED_MODE, OPT_WAIT_LIMIT_NS, OPT_SKIP_RANK, OPT_SCHED_THREADS,
- OPT_SCHED_RANKS_PER_CTA, OPT_BLOCKS) = range(1, 7)
+ OPT_SCHED_RANKS_PER_CTA, OPT_BLOCKS, OPT_SPLIT_DEPTH) = range(1, 8)
 
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libdpdr.so")
 

@@ -52,6 +52,7 @@ struct Plan {
     int skip_rank = -1;
     int sched_threads = 128;
     int sched_rpc = 0;         // ranks per CTA, 0 = auto
+    int split_depth = -1;      // cut depth of the split layout, -1 = auto
 
     // device memory: one allocation carved into the tables below
     char* dmem = nullptr;
@@ -113,7 +114,7 @@ int stage_pointers(Plan* P, const void* const* x, const void* const* y,
 // launchers
 int fused_launch(Plan* P, cudaStream_t s);      // fused.cu
 int fused_auto_mode(const Plan* P);             // fused.cu
-int fused_split_prepare(Plan* P, bool force);   // fused.cu
+int fused_split_prepare(Plan* P, bool force, int depth);  // fused.cu
 int schedule_launch(Plan* P, cudaStream_t s);   // schedule.cu
 int schedule_configure(Plan* P);                // schedule.cu
 

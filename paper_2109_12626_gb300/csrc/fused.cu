@@ -282,13 +282,21 @@ __device__ __forceinline__ void cp_async16(void* smem, const void* gmem)
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem)
                  : "memory");
 }
+__device__ __forceinline__ void cp_async4(void* smem, const void* gmem)
+{
+    const unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(s), "l"(gmem)
+                 : "memory");
+}
 __device__ __forceinline__ void cp_async_wait_all()
 {
     asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;\n" ::: "memory");
 }
 
-// rows of WU units: row i < p holds rank i's tile, row p the result
-template <class U, bool kAsync>
+// rows of WU units: row i < p holds rank i's tile, row p the result.
+// kVec: 16-byte units copied with 16-byte cp.async; otherwise single
+// elements copied word by word with 4-byte cp.async.
+template <class U, bool kVec, class Op>
 __device__ __forceinline__ void tile_body(const FusedArgs& a, int64_t u0,
                                           int wu, int lg_wu, typename U::T* tile)
 {
@@ -299,13 +307,17 @@ __device__ __forceinline__ void tile_body(const FusedArgs& a, int64_t u0,
     for (int idx = tid; idx < n; idx += bd) {
         const int i = idx >> lg_wu, c = idx & (WU - 1);
         if (c < wu) {
-            if constexpr (kAsync)
+            if constexpr (kVec) {
                 cp_async16(&tile[idx], rank_ptr(a.x, i) + (u0 + c) * 16);
-            else
-                tile[idx] = U::ld(rank_ptr(a.x, i), u0 + c);
+            } else {
+                const char* src = rank_ptr(a.x, i) + (u0 + c) * Op::kEsize;
+                uint32_t* dst = reinterpret_cast<uint32_t*>(&tile[idx]);
+#pragma unroll
+                for (int w = 0; w < Op::kEsize / 4; w++) cp_async4(dst + w, src + 4 * w);
+            }
         }
     }
-    if constexpr (kAsync) cp_async_wait_all();
+    cp_async_wait_all();
     __syncthreads();
     for (int l = 0; l < a.nlevels; l++) {
         const int beg = __ldg(a.level_off + l), end = __ldg(a.level_off + l + 1);
@@ -341,14 +353,14 @@ fused_tile_kernel(FusedArgs a)
     if (t < a.vec_tiles) {
         const int64_t u0 = t << a.lg_wu;
         const int wu = int(lmin(int64_t(1) << a.lg_wu, a.nvec - u0));
-        tile_body<VecUnit<Op>, true>(a, u0, wu, a.lg_wu, smem);
+        tile_body<VecUnit<Op>, true, Op>(a, u0, wu, a.lg_wu, smem);
     } else {
         // single elements: a row of a tile holds as many bytes as in the
         // vector tiles, i.e. 16/esize times more units
         const int lg = a.lg_wu + (Op::kEsize == 4 ? 2 : 0);
         const int64_t e0 = (t - a.vec_tiles) << lg;
         const int wu = int(lmin(int64_t(1) << lg, a.nscalar - e0));
-        tile_body<OneUnit<Op>, false>(a, a.scalar_base + e0, wu, lg,
+        tile_body<OneUnit<Op>, false, Op>(a, a.scalar_base + e0, wu, lg,
                                       reinterpret_cast<Elem<Op>*>(smem));
     }
 }
@@ -436,20 +448,26 @@ int fused_auto_mode(const Plan* P)
 
 // Split layout: cut depth s, subtree table, top-of-tree item list, rank
 // groups of the finish kernel, and the scratch rows of subtree values.
-int fused_split_prepare(Plan* P, bool force)
+// depth < 0 picks the shallowest cut that gives the first kernel enough
+// independent (subtree, column) work to fill the GPU.
+int fused_split_prepare(Plan* P, bool force, int depth)
 {
-    if (P->split_ready) return DPDR_OK;
     const int p = P->p;
-    if (P->max_depth < 3) return DPDR_OK;  // nothing worth splitting
+    if (p < 2) return DPDR_OK;  // one rank: nothing to split
     const int64_t units = std::max<int64_t>(1, P->m * int64_t(P->esize) / 16);
     const int64_t target = stream_target(P);
-    if (!force && units >= target) return DPDR_OK;  // auto never picks it
-    int s = 1;
-    for (; s < P->max_depth - 2; s++) {
-        int64_t n = 0;
-        for (int i = 0; i < p; i++) n += P->depth[i] == s;
-        if (n * units >= target) break;
+    int s = depth;
+    if (s < 0) {
+        s = 0;
+        for (; s < std::max(0, P->max_depth - 2); s++) {
+            int64_t n = 0;
+            for (int i = 0; i < p; i++) n += P->depth[i] == s;
+            if (n * units >= target) break;
+        }
     }
+    s = std::min(s, P->max_depth);
+    if (P->split_ready && P->split_s == s) return DPDR_OK;
+    if (!force && units >= target) return DPDR_OK;  // auto streams instead
     // scratch rows: one per depth-s subtree (first rank, root), one per node
     // above the cut (its own input, first = root); items in post-order
     std::vector<int2> seg, items;
@@ -462,6 +480,12 @@ int fused_split_prepare(Plan* P, bool force)
         items.push_back(make_int2(int(seg.size()), int(t)));
         seg.push_back(make_int2(lo, i));
     }
+    if (P->d_split) {
+        cudaFree(P->d_split);
+        P->d_split = nullptr;
+        P->d_split_bytes = 0;
+        P->split_ready = false;
+    }
     int64_t groups = std::min<int64_t>(p, std::max<int64_t>(1, (target + units - 1) / units));
     P->split_group = int((p + groups - 1) / groups);
     P->split_s = s;
@@ -473,6 +497,7 @@ int fused_split_prepare(Plan* P, bool force)
     const size_t bytes = o_part + size_t(P->part_stride) * seg.size();
     cudaError_t e = cudaMalloc(&P->d_split, bytes);
     if (e != cudaSuccess) {
+        P->d_split = nullptr;
         P->split_nseg = 0;
         return cuda_fail(e, "split layout: cudaMalloc");
     }
@@ -495,7 +520,7 @@ int fused_launch(Plan* P, cudaStream_t s)
     int mode = P->fused_mode ? P->fused_mode : fused_auto_mode(P);
     const int lg = tile_lg_wu(P);
     if (mode == 2 && lg < 0) return fail(DPDR_ERR_INVALID, "tile mode: p too large");
-    if (mode == 3 && !P->split_ready) return fail(DPDR_ERR_INVALID, "split mode: p too small");
+    if (mode == 3 && !P->split_ready) return fail(DPDR_ERR_INVALID, "split mode: p < 2");
 
     FusedArgs a;
     a.x = P->d_x;

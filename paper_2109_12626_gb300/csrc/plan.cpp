@@ -328,7 +328,7 @@ extern "C" dpdr_plan_t dpdr_plan(int p, int64_t m, dpdr_dtype dtype,
         return nullptr;
     }
     if (allocate(P) != DPDR_OK || schedule_configure(P) != DPDR_OK ||
-        fused_split_prepare(P, false) != DPDR_OK) {
+        fused_split_prepare(P, false, P->split_depth) != DPDR_OK) {
         free_plan(P);
         return nullptr;
     }
@@ -359,9 +359,9 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
     case DPDR_OPT_FUSED_MODE:
         if (v < 0 || v > 3) return fail(DPDR_ERR_INVALID, "fused mode: 0, 1, 2 or 3");
         if (v == 3) {
-            int rc = fused_split_prepare(P, true);
+            int rc = fused_split_prepare(P, true, P->split_depth);
             if (rc) return rc;
-            if (!P->split_ready) return fail(DPDR_ERR_INVALID, "split mode needs trees of depth >= 3");
+            if (!P->split_ready) return fail(DPDR_ERR_INVALID, "split mode needs p >= 2");
         }
         P->fused_mode = int(v);
         return DPDR_OK;
@@ -382,6 +382,11 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
         if (v < 0 || v > P->p) return fail(DPDR_ERR_INVALID, "ranks per CTA out of range");
         P->sched_rpc = int(v);
         return schedule_configure(P);
+    case DPDR_OPT_SPLIT_DEPTH: {
+        if (v < -1 || v > P->max_depth) return fail(DPDR_ERR_INVALID, "split depth out of range");
+        P->split_depth = int(v);
+        return fused_split_prepare(P, true, P->split_depth);
+    }
     case DPDR_OPT_BLOCKS: {
         if (v < 0) return fail(DPDR_ERR_INVALID, "b < 0");
         const int nb = clamp_b(P->m, v == 0 ? block_count_rule(P->p, P->m, 0) : v);
