@@ -263,7 +263,8 @@ def main(argv=None) -> int:
     ap.add_argument("--m", type=int, default=None, help="override m (sweeps)")
     ap.add_argument("--kernel", choices=("fused", "schedule"), default="fused")
     ap.add_argument("--b", type=int, default=None, help="pipeline blocks (schedule)")
-    ap.add_argument("--mode", type=int, default=0, help="fused layout: 0 auto, 1, 2")
+    ap.add_argument("--mode", type=int, default=0, help="fused layout: 0 auto, 1, 2, 3")
+    ap.add_argument("--split-depth", type=int, default=None, help="split layout cut depth")
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
@@ -298,6 +299,8 @@ def main(argv=None) -> int:
     xs = gen_device_inputs(w, dev)
     ys = [torch.empty_like(x) for x in xs]
     plan = pkg.Plan(p, m, kind, b)
+    if args.split_depth is not None:
+        plan.set(pkg.OPT_SPLIT_DEPTH, args.split_depth)
     if args.mode:
         plan.set(pkg.OPT_FUSED_MODE, args.mode)
     stream = torch.cuda.current_stream(dev)
@@ -313,15 +316,19 @@ def main(argv=None) -> int:
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(args.steps)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    bound = plan.bind(xs, ys)
+    go = bound.allreduce if args.kernel == "fused" else bound.allreduce_schedule
     barrier(world)
     torch.cuda.synchronize(dev)
+    torch.cuda.nvtx.range_push("dpdr_timed")
     start.record(stream)
     for k in range(args.steps):
         ev[k][0].record(stream)
-        run(xs, ys, stream)
+        go(stream)
         ev[k][1].record(stream)
     stop.record(stream)
     torch.cuda.synchronize(dev)
+    torch.cuda.nvtx.range_pop()
     barrier(world)
     clocks = sampler.stop()
     plan.sync(stream)
@@ -368,6 +375,7 @@ def main(argv=None) -> int:
                "sample": sample}
 
     info = plan.info()
+    launches_per_step = 2 if (args.kernel == "fused" and (args.mode or info["auto_mode"]) == 3) else 1
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
@@ -377,6 +385,7 @@ def main(argv=None) -> int:
         "config": {"workload": args.workload, "p": p, "m": m, "kind": kind,
                    "kernel": args.kernel, "b": info["b"],
                    "fused_mode": args.mode or info["auto_mode"],
+                   "split_depth": info["split_depth"] if (args.mode or info["auto_mode"]) == 3 else None,
                    "bytes_per_step": algo_bytes,
                    "l2": "inputs larger than L2 (%.1f GB), no flush" % (algo_bytes / 2e9)
                    if algo_bytes / 2 > 129e6 else "working set fits L2: warm-cache number",
@@ -388,7 +397,7 @@ def main(argv=None) -> int:
                      "kernel_ms": round(avg_launch, 4)},
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": args.steps,
+        "gpu_launches": args.steps * launches_per_step,
         "clocks": clocks,
     }
     if rank == 0:

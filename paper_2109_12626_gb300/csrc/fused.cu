@@ -344,24 +344,34 @@ __device__ __forceinline__ void tile_body(const FusedArgs& a, int64_t u0,
     }
 }
 
+// smallest power-of-two exponent with 2^lg >= w
+__device__ __forceinline__ int ceil_lg(int w)
+{
+    int lg = 0;
+    while ((1 << lg) < w) lg++;
+    return lg;
+}
+
 template <class Op>
 __global__ void __launch_bounds__(kTileThreads)
 fused_tile_kernel(FusedArgs a)
 {
     extern __shared__ uint4 smem[];
     const int64_t t = blockIdx.x;
+    // a narrow last tile (small m) is packed with a row stride of its own
+    // width, so no thread walks empty columns
     if (t < a.vec_tiles) {
         const int64_t u0 = t << a.lg_wu;
         const int wu = int(lmin(int64_t(1) << a.lg_wu, a.nvec - u0));
-        tile_body<VecUnit<Op>, true, Op>(a, u0, wu, a.lg_wu, smem);
+        tile_body<VecUnit<Op>, true, Op>(a, u0, wu, ceil_lg(wu), smem);
     } else {
         // single elements: a row of a tile holds as many bytes as in the
         // vector tiles, i.e. 16/esize times more units
         const int lg = a.lg_wu + (Op::kEsize == 4 ? 2 : 0);
         const int64_t e0 = (t - a.vec_tiles) << lg;
         const int wu = int(lmin(int64_t(1) << lg, a.nscalar - e0));
-        tile_body<OneUnit<Op>, false, Op>(a, a.scalar_base + e0, wu, lg,
-                                      reinterpret_cast<Elem<Op>*>(smem));
+        tile_body<OneUnit<Op>, false, Op>(a, a.scalar_base + e0, wu, ceil_lg(wu),
+                                          reinterpret_cast<Elem<Op>*>(smem));
     }
 }
 
@@ -437,13 +447,28 @@ int tile_lg_wu(const Plan* P)
 // Threads the streaming layouts want in flight to cover HBM latency.
 static int64_t stream_target(const Plan* P) { return int64_t(P->num_sms) * 1024; }
 
+// Layout choice, from measurements on GB300:
+//  * deep trees (p >= 128) with at least 8192 column units: the split layout,
+//    whose read phase (first kernel) and write phase (second kernel) keep
+//    HBM traffic one-directional; it beats column streaming from m = 2^15 up
+//    to the largest sizes at p = 1152;
+//  * otherwise column streaming once there are enough columns to fill the
+//    GPU, and the shared-memory tile below that.
 int fused_auto_mode(const Plan* P)
 {
     const int64_t units = P->m * int64_t(P->esize) / 16;
-    // column streaming needs enough independent columns to fill every SM
+    if (P->p >= 128 && units >= 8192 && P->split_ready) return 3;
     if (units >= stream_target(P)) return 1;
-    if (P->split_nseg > 0 && units * P->split_nseg >= int64_t(P->num_sms) * 256) return 3;
-    return tile_lg_wu(P) < 0 ? (P->split_nseg > 0 ? 3 : 1) : 2;
+    if (tile_lg_wu(P) >= 0) return 2;
+    return P->split_ready ? 3 : 1;
+}
+
+// Whether the automatic choice can be the split layout (then the plan
+// prepares it up front).
+static bool split_wanted(const Plan* P)
+{
+    const int64_t units = P->m * int64_t(P->esize) / 16;
+    return P->p >= 128 && units >= 8192;
 }
 
 // Split layout: cut depth s, subtree table, top-of-tree item list, rank
@@ -456,18 +481,22 @@ int fused_split_prepare(Plan* P, bool force, int depth)
     if (p < 2) return DPDR_OK;  // one rank: nothing to split
     const int64_t units = std::max<int64_t>(1, P->m * int64_t(P->esize) / 16);
     const int64_t target = stream_target(P);
+    // automatic cut: the shallowest depth whose subtrees give the first
+    // kernel four times the columns the GPU needs in flight, but no deeper
+    // than a third of the tree height (the second kernel's sequential walk
+    // over the nodes above the cut grows as 2^(s+1))
     int s = depth;
     if (s < 0) {
-        s = 0;
-        for (; s < std::max(0, P->max_depth - 2); s++) {
+        const int cap = std::max(1, P->max_depth / 3);
+        for (s = 0; s < cap; s++) {
             int64_t n = 0;
             for (int i = 0; i < p; i++) n += P->depth[i] == s;
-            if (n * units >= target) break;
+            if (n * units >= 4 * target) break;
         }
     }
     s = std::min(s, P->max_depth);
     if (P->split_ready && P->split_s == s) return DPDR_OK;
-    if (!force && units >= target) return DPDR_OK;  // auto streams instead
+    if (!force && !split_wanted(P)) return DPDR_OK;
     // scratch rows: one per depth-s subtree (first rank, root), one per node
     // above the cut (its own input, first = root); items in post-order
     std::vector<int2> seg, items;
