@@ -176,7 +176,7 @@ def kernel_source_hash(kernel: str) -> str:
 def profiled_traffic(kernel: str, wname: str, units: int) -> float | None:
     """DRAM bytes per launch from the committed ncu summary, scaled to the
     units of this launch; None if the kernel changed since the capture."""
-    path = os.path.join(ROOT, "profiles", "traffic.json")
+    path = os.path.join(ROOT, "profiles", "traffic.json")  # ncu figures, not code
     try:
         with open(path) as f:
             rec = json.load(f)[kernel][wname]
