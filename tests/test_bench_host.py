@@ -1,0 +1,90 @@
+"""bench.py's host-side logic without a GPU: the max-over-ranks timing and
+barrier with two gloo ranks on the CPU (the N > 1 replica path), the clock
+sample parsing, the measured-traffic lookup, and the reference arm (the CPU
+oracle on a bounded sample)."""
+import json
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+import bench  # noqa: E402
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, q):
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    bench.barrier(world)
+    t = bench.max_over_ranks(10.0 + 5.0 * rank, world)   # rank 1 is slower
+    bench.barrier(world)
+    q.put((rank, t))
+    dist.destroy_process_group()
+
+
+def test_max_over_ranks_gloo_two_ranks():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_main, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(120)
+        assert p.exitcode == 0
+    got = dict(q.get(timeout=10) for _ in range(2))
+    assert got == {0: 15.0, 1: 15.0}
+
+
+def test_single_rank_needs_no_process_group():
+    assert bench.max_over_ranks(3.5, 1) == 3.5
+    bench.barrier(1)
+
+
+def test_clock_summary():
+    csv = "\n".join([
+        "0, 2070, 2070, 900.5, 0x0, Not Active, Not Active, Not Active, Not Active",
+        "0, 2055, 2070, 1100.0, 0x4, Not Active, Not Active, Not Active, Active",
+        "0, 1980, 2070, 95.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+    ])
+    c = bench.summarize_clocks(csv)
+    assert c["sm_max_mhz"] == 2070 and c["samples"] == 2   # idle sample dropped
+    assert c["sm_mhz"] == pytest.approx((2070 + 2055) / 2)
+    assert c["reasons"] == ["sw_power_cap"]
+    assert bench.summarize_clocks("") is None
+
+
+def test_profiled_traffic_tracks_the_kernel_source():
+    rec = json.load(open(os.path.join(ROOT, "profiles", "traffic.json")))
+    for kernel, table in rec.items():
+        for wname, r in table.items():
+            got = bench.profiled_traffic(kernel, wname, 1000)
+            if r["source_hash"] == bench.kernel_source_hash(kernel):
+                assert got == pytest.approx(1000 * r["bytes_per_unit"])
+            else:
+                assert got is None  # stale counters are not reported
+
+
+def test_reference_arm_prints_one_json_line():
+    out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl",
+                          "reference", "--workload", "p7_m1000_int32", "--steps", "2",
+                          "--warmup", "3"], capture_output=True, text=True, timeout=300)
+    assert out.returncode == 0, out.stderr
+    lines = [l for l in out.stdout.splitlines() if l.strip()]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["unit"] == "GB/s" and d["value"] > 0
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] == 1
+    assert d["e2e"]["h2d_bytes_per_step"] == 0
