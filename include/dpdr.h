@@ -129,7 +129,11 @@ int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
  *                             fit co-resident)
  *   DPDR_OPT_BLOCKS           change b (same rules as dpdr_plan's b)
  *   DPDR_OPT_SPLIT_DEPTH      tree depth at which the split layout cuts
- *                             the ranks into subtrees (-1 = automatic) */
+ *                             the ranks into subtrees (-1 = automatic)
+ *   DPDR_OPT_SCHED_SLICES     CTAs per virtual rank in the schedule kernel,
+ *                             each owning one column slice of every block
+ *                             (0 = as many as fit co-resident, slices of at
+ *                             least 1024 elements, at most 64) */
 enum {
     DPDR_OPT_FUSED_MODE = 1,
     DPDR_OPT_WAIT_LIMIT_NS = 2,
@@ -137,7 +141,8 @@ enum {
     DPDR_OPT_SCHED_THREADS = 4,
     DPDR_OPT_SCHED_RANKS_PER_CTA = 5,
     DPDR_OPT_BLOCKS = 6,
-    DPDR_OPT_SPLIT_DEPTH = 7
+    DPDR_OPT_SPLIT_DEPTH = 7,
+    DPDR_OPT_SCHED_SLICES = 8
 };
 int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
 
@@ -147,7 +152,8 @@ int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
  *   [8] 1 if the last dpdr_allreduce ran the 16-byte vector path
  *   [9] split layout cut depth  [10] its scratch rows (subtrees plus nodes
  *   above the cut)  [11] ranks per store
- *   group of its second kernel (0 when the split layout is not prepared) */
+ *   group of its second kernel (0 when the split layout is not prepared)
+ *   [12] CTAs per rank (column slices) of the schedule kernel */
 int dpdr_plan_info(dpdr_plan_t plan, int64_t* info, int n);
 
 /* Releases the plan's device and host memory.  The caller must first make

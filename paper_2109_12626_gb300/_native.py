@@ -17,7 +17,7 @@ DPDR_OP_SUM, DPDR_OP_MATMUL = 0, 1
 (DPDR_OK, DPDR_ERR_INVALID, DPDR_ERR_CUDA, DPDR_ERR_TIMEOUT,
  DPDR_ERR_NOT_COOPERATIVE, DPDR_ERR_OOM) = range(6)
 (OPT_FUSED_MODE, OPT_WAIT_LIMIT_NS, OPT_SKIP_RANK, OPT_SCHED_THREADS,
- OPT_SCHED_RANKS_PER_CTA, OPT_BLOCKS, OPT_SPLIT_DEPTH) = range(1, 8)
+ OPT_SCHED_RANKS_PER_CTA, OPT_BLOCKS, OPT_SPLIT_DEPTH, OPT_SCHED_SLICES) = range(1, 9)
 
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libdpdr.so")
 
@@ -174,12 +174,12 @@ class Plan:
         return out
 
     def info(self) -> dict:
-        v = np.zeros(12, np.int64)
-        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), 12),
+        v = np.zeros(13, np.int64)
+        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), 13),
                "dpdr_plan_info")
         keys = ("p", "m", "b", "max_depth", "auto_mode", "sched_ctas",
                 "sched_ranks_per_cta", "scratch_bytes", "vector_path",
-                "split_depth", "split_subtrees", "split_group")
+                "split_depth", "split_subtrees", "split_group", "sched_slices")
         return {k: int(x) for k, x in zip(keys, v)}
 
     def set(self, key: int, value: int) -> None:

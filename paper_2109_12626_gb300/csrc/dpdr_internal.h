@@ -52,6 +52,7 @@ struct Plan {
     int skip_rank = -1;
     int sched_threads = 128;
     int sched_rpc = 0;         // ranks per CTA, 0 = auto
+    int sched_slices = 0;      // CTAs per rank (column slices), 0 = auto
     int split_depth = -1;      // cut depth of the split layout, -1 = auto
 
     // device memory: one allocation carved into the tables below
@@ -63,12 +64,13 @@ struct Plan {
     LevelNode* d_levels = nullptr;
     int* d_level_off = nullptr;
     int* d_tables = nullptr;         // parent, child0, child1, depth: 4 x [p]
-    uint32_t* d_ctrl = nullptr;      // up[p], down[p], abort word
+    uint32_t* d_ctrl = nullptr;      // up[G*p], down[G*p], abort word (in d_sched)
     uint32_t* d_err = nullptr;       // 4 words: status, rank, round, step
     char* d_ring = nullptr;          // dual-root exchange slots: [2][2][slot]
     size_t ring_slot_bytes = 0;
-    int* d_cta_first = nullptr;      // schedule CTA -> first rank (+1 entry)
-    int cta_capacity = 0;            // entries reserved in d_cta_first
+    int* d_cta_first = nullptr;      // schedule chunk -> first rank (+1 entry)
+    char* d_sched = nullptr;         // own allocation: counters + chunk table
+    size_t d_sched_bytes = 0;
 
     // rank-pointer staging (pinned host), copied to d_x / d_y when they change
     const void** h_ptrs = nullptr;   // [2p]
@@ -93,6 +95,7 @@ struct Plan {
     // facts
     int last_vector_path = 0;
     int sched_ctas = 0, sched_ranks_per_cta = 0;
+    int sched_slices_used = 1, sched_chunks = 1;
 };
 
 // host-side builders (plan.cpp)

@@ -210,6 +210,7 @@ static void free_plan(Plan* P)
     if (!P) return;
     if (P->staged) cudaEventDestroy(P->staged);
     if (P->d_split) cudaFree(P->d_split);
+    if (P->d_sched) cudaFree(P->d_sched);
     if (P->h_ptrs) cudaFreeHost(P->h_ptrs);
     if (P->dmem) cudaFree(P->dmem);
     delete P;
@@ -227,7 +228,6 @@ static int allocate(Plan* P)
 {
     const int p = P->p;
     P->ring_slot_bytes = ring_slot(P);
-    P->cta_capacity = 2 * p + 2;
     size_t off = 0;
     auto carve = [&](size_t bytes) {
         size_t o = off;
@@ -239,9 +239,7 @@ static int allocate(Plan* P)
     const size_t o_lv = carve(sizeof(LevelNode) * std::max<size_t>(P->levels.size(), 1));
     const size_t o_lo = carve(sizeof(int) * P->level_off.size());
     const size_t o_tab = carve(sizeof(int) * 4 * size_t(p));
-    const size_t o_ctrl = carve(sizeof(uint32_t) * (2 * size_t(p) + 1));
     const size_t o_err = carve(sizeof(uint32_t) * 4);
-    const size_t o_cta = carve(sizeof(int) * size_t(P->cta_capacity + 1));
     const size_t o_ring = carve(4 * P->ring_slot_bytes);
     P->dmem_bytes = off;
     cudaError_t e = cudaMalloc(&P->dmem, off);
@@ -253,9 +251,7 @@ static int allocate(Plan* P)
     P->d_levels = reinterpret_cast<LevelNode*>(base + o_lv);
     P->d_level_off = reinterpret_cast<int*>(base + o_lo);
     P->d_tables = reinterpret_cast<int*>(base + o_tab);
-    P->d_ctrl = reinterpret_cast<uint32_t*>(base + o_ctrl);
     P->d_err = reinterpret_cast<uint32_t*>(base + o_err);
-    P->d_cta_first = reinterpret_cast<int*>(base + o_cta);
     P->d_ring = base + o_ring;
 
     std::vector<int> tab(size_t(4) * p);
@@ -382,6 +378,10 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
         if (v < 0 || v > P->p) return fail(DPDR_ERR_INVALID, "ranks per CTA out of range");
         P->sched_rpc = int(v);
         return schedule_configure(P);
+    case DPDR_OPT_SCHED_SLICES:
+        if (v < 0 || v > 1024) return fail(DPDR_ERR_INVALID, "slices: 0..1024");
+        P->sched_slices = int(v);
+        return schedule_configure(P);
     case DPDR_OPT_SPLIT_DEPTH: {
         if (v < -1 || v > P->max_depth) return fail(DPDR_ERR_INVALID, "split depth out of range");
         P->split_depth = int(v);
@@ -398,7 +398,7 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
             return fail(DPDR_ERR_INVALID,
                         "fewer blocks than the plan was built for: make a new plan");
         P->b = nb;
-        return DPDR_OK;
+        return schedule_configure(P);
     }
     default:
         return fail(DPDR_ERR_INVALID, "unknown option");
@@ -412,7 +412,8 @@ extern "C" int dpdr_plan_info(dpdr_plan_t h, int64_t* info, int n)
     const int64_t v[] = {P->p, P->m, P->b, P->max_depth, fused_auto_mode(P),
                          P->sched_ctas, P->sched_ranks_per_cta,
                          int64_t(P->dmem_bytes + P->d_split_bytes), P->last_vector_path,
-                         P->split_s, P->split_nseg, P->split_group};
+                         P->split_s, P->split_nseg, P->split_group,
+                         P->sched_slices_used};
     const int k = int(sizeof v / sizeof v[0]);
     for (int i = 0; i < n; i++) info[i] = i < k ? v[i] : 0;
     return DPDR_OK;

@@ -26,7 +26,10 @@
 // k: the data dependencies of the algorithm order every reuse, so a sender
 // never waits for its receiver.
 //
-// CTAs own contiguous rank ranges that never straddle the two trees and run
+// A virtual rank is served by a group of nslices CTAs, one per column slice
+// of every pipeline block; slices are independent copies of the schedule
+// (their own counters), since (.) acts column by column.  CTAs own
+// contiguous rank ranges that never straddle the two trees and run
 // their ranks in increasing order inside each round.  Every wait is then on
 // a lower rank of the same round, on an earlier round, or (r0 only) on the
 // dual r1 whose partial depends on tree 1 alone, so with all CTAs resident
@@ -63,6 +66,8 @@ struct SchedArgs {
     int64_t wait_ns;
     int skip_rank;
     int vec;
+    int nslices;   // CTAs per rank: each owns one column slice of every block
+    int nchunks;   // rank ranges (CTA index = slice * nchunks + chunk)
 };
 
 __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p)
@@ -91,6 +96,17 @@ __device__ __forceinline__ uint64_t now_ns()
 __device__ __forceinline__ int64_t blk_start(const SchedArgs& a, int j)
 {
     return int64_t(j) * a.q + lmin(j, a.rem);
+}
+
+// Start of column slice g (of nslices) of the element range [s, e): even
+// shares, inner boundaries rounded down to a 16-byte vector boundary.
+template <int EPV>
+__device__ __forceinline__ int64_t slice_at(const SchedArgs& a, int64_t s, int64_t e, int g)
+{
+    if (g <= 0) return s;
+    if (g >= a.nslices) return e;
+    const int64_t b = (s + (e - s) * g / a.nslices) / EPV * EPV;
+    return b < s ? s : b;
 }
 
 // Thread 0 waits for *ctr >= target within the plan's time bound; the CTA
@@ -198,8 +214,11 @@ __device__ __forceinline__ char* ring_base(const SchedArgs& a, int side, int j,
 }
 
 template <class Op>
-__device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j)
+__device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j, int g)
 {
+    constexpr int EPV = Op::kEpv;
+    uint32_t* const up = a.up + int64_t(g) * a.p;      // this slice's counters
+    uint32_t* const down = a.down + int64_t(g) * a.p;
     const int d = __ldg(a.depth + i);
     const int c0 = __ldg(a.child0 + i), c1 = __ldg(a.child1 + i);
     const int par = __ldg(a.parent + i);
@@ -208,9 +227,10 @@ __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j)
     const bool root = par < 0;
     const bool paired_root = root && a.p >= 2;
     const bool inb = j < a.b;
-    const int64_t s = inb ? blk_start(a, j) : 0, e = inb ? blk_start(a, j + 1) : 0;
+    const int64_t bs = inb ? blk_start(a, j) : 0, be = inb ? blk_start(a, j + 1) : 0;
+    const int64_t s = slice_at<EPV>(a, bs, be, g), e = slice_at<EPV>(a, bs, be, g + 1);
     const int side = (i == a.r0) ? 0 : 1;
-    char* dst = paired_root ? ring_base(a, side, j, s, Op::kEpv, Op::kEsize) : yi;
+    char* dst = paired_root ? ring_base(a, side, j, bs, Op::kEpv, Op::kEsize) : yi;
 
     // steps 1 and 2: child_0 then child_1; the send half (final block
     // j-(d+1)) is read by the child itself from y_i once down[i] covers it
@@ -218,7 +238,7 @@ __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j)
     for (int k = 0; k < 2; k++) {
         const int c = k ? c1 : c0;
         if (c < 0 || !inb) continue;
-        if (!cta_wait(a, a.up + c, uint32_t(j + 1), i, j, k)) return false;
+        if (!cta_wait(a, up + c, uint32_t(j + 1), i, j, k)) return false;
         const bool leaf = __ldg(a.child0 + c) < 0;
         const char* src = leaf
             ? reinterpret_cast<const char*>(__ldg(reinterpret_cast<const unsigned long long*>(a.x) + c))
@@ -234,15 +254,15 @@ __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j)
             block_op<Op>(a, dst, nullptr, xi, s, e);
             __syncthreads();
         }
-        publish(a, a.up + i, uint32_t(j + 1), i);
+        publish(a, up + i, uint32_t(j + 1), i);
         const int du = (i == a.r0) ? a.r1 : a.r0;
-        if (!cta_wait(a, a.up + du, uint32_t(j + 1), i, j, 2)) return false;
-        const char* other = ring_base(a, 1 - side, j, s, Op::kEpv, Op::kEsize);
+        if (!cta_wait(a, up + du, uint32_t(j + 1), i, j, 2)) return false;
+        const char* other = ring_base(a, 1 - side, j, bs, Op::kEpv, Op::kEsize);
         if (i == a.r0)
             block_op<Op>(a, yi, dst, other, s, e);  // lower root: Y[j] (.) t
         else
             block_op<Op>(a, yi, other, dst, s, e);  // higher root: t (.) Y[j]
-        publish(a, a.down + i, uint32_t(j + 1), i);
+        publish(a, down + i, uint32_t(j + 1), i);
         return true;
     }
     if (root) {  // p == 1: one processor, y = x
@@ -254,13 +274,14 @@ __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j)
     }
     // step 3 elsewhere: partial Y[j] up (in y_i, or x_i for a leaf), final
     // Y[j-d] down from the parent
-    if (inb) publish(a, a.up + i, uint32_t(j + 1), i);
+    if (inb) publish(a, up + i, uint32_t(j + 1), i);
     const int kf = j - d;
     if (kf >= 0 && kf < a.b) {
-        if (!cta_wait(a, a.down + par, uint32_t(kf + 1), i, j, 3)) return false;
+        if (!cta_wait(a, down + par, uint32_t(kf + 1), i, j, 3)) return false;
         const char* yp = reinterpret_cast<const char*>(__ldg(reinterpret_cast<const unsigned long long*>(a.y) + par));
-        block_op<Op>(a, yi, nullptr, yp, blk_start(a, kf), blk_start(a, kf + 1));
-        publish(a, a.down + i, uint32_t(kf + 1), i);
+        const int64_t ks = blk_start(a, kf), ke = blk_start(a, kf + 1);
+        block_op<Op>(a, yi, nullptr, yp, slice_at<EPV>(a, ks, ke, g), slice_at<EPV>(a, ks, ke, g + 1));
+        publish(a, down + i, uint32_t(kf + 1), i);
     }
     return true;
 }
@@ -268,14 +289,15 @@ __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j)
 template <class Op>
 __global__ void __launch_bounds__(kSchedMaxThreads, 4) schedule_kernel(SchedArgs a)
 {
-    const int first = __ldg(a.cta_first + blockIdx.x);
-    const int last = __ldg(a.cta_first + blockIdx.x + 1);
+    const int g = blockIdx.x / a.nchunks, chunk = blockIdx.x % a.nchunks;
+    const int first = __ldg(a.cta_first + chunk);
+    const int last = __ldg(a.cta_first + chunk + 1);
     int rounds = 0;
     for (int i = first; i < last; i++) rounds = max(rounds, a.b + __ldg(a.depth + i));
     for (int j = 0; j <= rounds; j++) {
         for (int i = first; i < last; i++) {
             if (j > a.b + __ldg(a.depth + i)) continue;
-            if (!run_round<Op>(a, i, j)) return;
+            if (!run_round<Op>(a, i, j, g)) return;
         }
     }
 }
@@ -297,8 +319,11 @@ const void* kernel_for(int dtype)
 
 }  // namespace
 
-// Choose ranks per CTA so that every CTA can be resident at once, with CTA
-// boundaries on the tree boundary, and upload the CTA -> rank table.
+// Choose the CTA layout so that every CTA can be resident at once: ranks per
+// CTA (rank ranges never straddle the trees) and, when the GPU has room for
+// more CTAs than ranks, CTAs per rank (column slices of at least 1024
+// elements).  Allocates the counters for that many slices and uploads the
+// chunk -> first rank table.
 int schedule_configure(Plan* P)
 {
     int occ = 0;
@@ -317,9 +342,29 @@ int schedule_configure(Plan* P)
     for (int lo = 0; lo < n0; lo += R) first.push_back(lo);
     for (int lo = n0; lo < P->p; lo += R) first.push_back(lo);
     first.push_back(P->p);
-    P->sched_ctas = int(first.size()) - 1;
+    const int nchunks = int(first.size()) - 1;
+    int G = P->sched_slices;
+    if (G == 0) {
+        const int64_t blk = (P->m + P->b - 1) / std::max(P->b, 1);
+        const int64_t room = std::max<int64_t>(1, kmax / nchunks);
+        G = int(std::max<int64_t>(1, std::min<int64_t>({room, blk / 1024, 64})));
+    }
+    const size_t words = 2 * size_t(P->p) * G + 1;
+    const size_t bytes = (words * sizeof(uint32_t) + 255) / 256 * 256 + sizeof(int) * first.size();
+    if (bytes > P->d_sched_bytes) {
+        if (P->d_sched) cudaFree(P->d_sched);
+        P->d_sched = nullptr;
+        P->d_sched_bytes = 0;
+        e = cudaMalloc(&P->d_sched, bytes);
+        if (e != cudaSuccess) return cuda_fail(e, "schedule counters: cudaMalloc");
+        P->d_sched_bytes = bytes;
+    }
+    P->d_ctrl = reinterpret_cast<uint32_t*>(P->d_sched);
+    P->d_cta_first = reinterpret_cast<int*>(P->d_sched + (words * sizeof(uint32_t) + 255) / 256 * 256);
+    P->sched_slices_used = G;
+    P->sched_chunks = nchunks;
+    P->sched_ctas = nchunks * G;
     P->sched_ranks_per_cta = R;
-    if (P->sched_ctas > P->cta_capacity) return fail(DPDR_ERR_INVALID, "too many CTAs");
     e = cudaMemcpy(P->d_cta_first, first.data(), sizeof(int) * first.size(),
                    cudaMemcpyHostToDevice);
     if (e != cudaSuccess) return cuda_fail(e, "schedule table upload");
@@ -337,9 +382,10 @@ int schedule_launch(Plan* P, cudaStream_t s)
     a.child1 = P->d_tables + 2 * P->p;
     a.depth = P->d_tables + 3 * P->p;
     a.cta_first = P->d_cta_first;
+    const int64_t cw = int64_t(P->p) * P->sched_slices_used;
     a.up = P->d_ctrl;
-    a.down = P->d_ctrl + P->p;
-    a.abort_flag = P->d_ctrl + 2 * P->p;
+    a.down = P->d_ctrl + cw;
+    a.abort_flag = P->d_ctrl + 2 * cw;
     a.err = P->d_err;
     a.ring = P->d_ring;
     a.ring_slot = int64_t(P->ring_slot_bytes);
@@ -353,8 +399,10 @@ int schedule_launch(Plan* P, cudaStream_t s)
     a.wait_ns = P->wait_ns;
     a.skip_rank = P->skip_rank;
     a.vec = P->last_vector_path;
+    a.nslices = P->sched_slices_used;
+    a.nchunks = P->sched_chunks;
 
-    cudaError_t e = cudaMemsetAsync(P->d_ctrl, 0, sizeof(uint32_t) * (2 * size_t(P->p) + 1), s);
+    cudaError_t e = cudaMemsetAsync(P->d_ctrl, 0, sizeof(uint32_t) * (2 * size_t(cw) + 1), s);
     if (e != cudaSuccess) return cuda_fail(e, "schedule counter reset");
     void* args[] = {&a};
     e = cudaLaunchCooperativeKernel(kernel_for(P->dtype), dim3(P->sched_ctas),
@@ -566,6 +614,8 @@ int schedule_noalloc(int p, int64_t m, int dtype, int op, int b, const void* con
     a.wait_ns = 4000000000LL;
     a.skip_rank = -1;
     a.vec = vec;
+    a.nslices = 1;
+    a.nchunks = nctas;
     void* args[] = {&a};
     e = cudaLaunchCooperativeKernel(kernel_for(dtype), dim3(nctas), dim3(kNoAllocThreads), args, 0, s);
     if (e == cudaErrorCooperativeLaunchTooLarge) {

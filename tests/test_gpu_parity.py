@@ -235,3 +235,24 @@ def test_invalid_arguments(pkg):
             plan.set(N.OPT_FUSED_MODE, 5)
         with pytest.raises(DpdrError):
             plan.set(999, 1)
+
+
+@pytest.mark.parametrize("kind,p,m,b,slices", [
+    ("float32", 32, 65541, 4, 7), ("int32", 7, 1000, 4, 3), ("mat2x2u32", 36, 4099, 16, 5),
+    ("float32", 1152, 4099, 3, 2), ("int32", 2, 333, 1, 64), ("float32", 1, 17, 2, 3)])
+@pytest.mark.parametrize("layout", ["aligned", "in_place", "four_byte"])
+def test_schedule_column_slices(pkg, orc, kind, p, m, b, slices, layout):
+    """Several CTAs per virtual rank, each running the schedule on its own
+    column slice of every block, give the same bits."""
+    x = host_inputs(kind, 61, p, m)
+    want = _want(orc, x, kind)
+    dev = torch.device("cuda:0")
+    pad = 1 if layout == "four_byte" else 0
+    xs, keep = to_device(x, kind, dev, pad_front=pad)
+    ys, keep_y = (xs, None) if layout == "in_place" else empty_like_ranks(xs, pad_front=pad)
+    with pkg.Plan(p, m, kind, b) as plan:
+        plan.set(pkg.OPT_SCHED_SLICES, slices)
+        assert plan.info()["sched_slices"] == slices
+        plan.allreduce_schedule(xs, ys)
+        plan.sync()
+    _check_all(ys, want)
