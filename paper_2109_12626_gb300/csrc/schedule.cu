@@ -333,10 +333,12 @@ int schedule_configure(Plan* P)
     const int64_t kmax = int64_t(occ) * P->num_sms;
     const int n0 = P->p / 2, n1 = P->p - n0;
     auto ctas = [&](int r) { return (n0 + r - 1) / r + (n1 + r - 1) / r; };
+    // with a fixed number of slices, ranks per CTA must make room for them
+    const int64_t per_chunk = std::max(1, P->sched_slices);
     int R = P->sched_rpc;
     if (R == 0) {
         R = 1;
-        while (R < P->p && ctas(R) > kmax) R++;
+        while (R < P->p && ctas(R) * per_chunk > kmax) R++;
     }
     std::vector<int> first;
     for (int lo = 0; lo < n0; lo += R) first.push_back(lo);
