@@ -133,7 +133,10 @@ int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
  *   DPDR_OPT_SCHED_SLICES     CTAs per virtual rank in the schedule kernel,
  *                             each owning one column slice of every block
  *                             (0 = as many as fit co-resident, slices of at
- *                             least 1024 elements, at most 64) */
+ *                             least 1024 elements, at most 64)
+ *   DPDR_OPT_HOST_CHUNK_BYTES bytes of rank data per column chunk of
+ *                             dpdr_allreduce_host's pipeline (default 2^30,
+ *                             minimum 4096) */
 enum {
     DPDR_OPT_FUSED_MODE = 1,
     DPDR_OPT_WAIT_LIMIT_NS = 2,
@@ -142,7 +145,8 @@ enum {
     DPDR_OPT_SCHED_RANKS_PER_CTA = 5,
     DPDR_OPT_BLOCKS = 6,
     DPDR_OPT_SPLIT_DEPTH = 7,
-    DPDR_OPT_SCHED_SLICES = 8
+    DPDR_OPT_SCHED_SLICES = 8,
+    DPDR_OPT_HOST_CHUNK_BYTES = 9
 };
 int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
 
@@ -182,10 +186,16 @@ int dpdr_allreduce(dpdr_plan_t plan, const void* const* x, void* const* y,
 int dpdr_allreduce_schedule(dpdr_plan_t plan, const void* const* x,
                             void* const* y, dpdr_stream_t stream);
 
-/* Host buffers end to end: copies x_host[i] (pinned or pageable host
- * memory) into the device buffers x_dev[i], runs dpdr_allreduce into y_dev,
- * and copies y_dev[i] back into y_host[i], all on stream.  All four are
- * host arrays of p pointers. */
+/* Host buffers end to end: copies x_host[i] into the device buffers
+ * x_dev[i], runs the fused kernel into y_dev, and copies y_dev[i] back into
+ * y_host[i].  All four are host arrays of p pointers; the device buffers
+ * follow dpdr_allreduce's rules.  The columns are cut into chunks (about
+ * 1 GB of rank data each) that flow through a pipeline: copies in on one
+ * plan-owned stream, the kernel on `stream`, copies out on another, so the
+ * two copy directions and the kernel overlap (with pinned host memory;
+ * pageable memory works but does not overlap).  The whole call is ordered
+ * after earlier work on `stream`, and later work on `stream` waits for its
+ * last copy. */
 int dpdr_allreduce_host(dpdr_plan_t plan, const void* const* x_host,
                         void* const* y_host, void* const* x_dev,
                         void* const* y_dev, dpdr_stream_t stream);

@@ -17,7 +17,8 @@ DPDR_OP_SUM, DPDR_OP_MATMUL = 0, 1
 (DPDR_OK, DPDR_ERR_INVALID, DPDR_ERR_CUDA, DPDR_ERR_TIMEOUT,
  DPDR_ERR_NOT_COOPERATIVE, DPDR_ERR_OOM) = range(6)
 (OPT_FUSED_MODE, OPT_WAIT_LIMIT_NS, OPT_SKIP_RANK, OPT_SCHED_THREADS,
- OPT_SCHED_RANKS_PER_CTA, OPT_BLOCKS, OPT_SPLIT_DEPTH, OPT_SCHED_SLICES) = range(1, 9)
+ OPT_SCHED_RANKS_PER_CTA, OPT_BLOCKS, OPT_SPLIT_DEPTH, OPT_SCHED_SLICES,
+ OPT_HOST_CHUNK_BYTES) = range(1, 10)
 
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libdpdr.so")
 

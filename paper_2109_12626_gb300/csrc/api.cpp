@@ -124,6 +124,59 @@ extern "C" int dpdr_allreduce_schedule(dpdr_plan_t h, const void* const* x,
     return schedule_launch(P, s);
 }
 
+// Column chunks of about host_chunk bytes of rank data (default 1 GB), each
+// row piece at least min(2 MB, host_chunk) so copies stay large, at most 64
+// chunks; chunk starts on 256-column boundaries (16-byte aligned).
+static int pipe_prepare(Plan* P, void* const* x_dev, void* const* y_dev, bool vec)
+{
+    const int p = P->p;
+    const int64_t es = int64_t(P->esize);
+    const int64_t row_min = std::min<int64_t>(int64_t(2) << 20, P->host_chunk);
+    int64_t cols = std::max<int64_t>(row_min / es, P->host_chunk / (p * es));
+    cols = std::max<int64_t>(cols, (P->m + 63) / 64);
+    cols = (cols + 255) / 256 * 256;
+    const int chunks = int((P->m + cols - 1) / cols);
+    cudaError_t e;
+    if (!P->pipe_in) {
+        e = cudaStreamCreateWithFlags(&P->pipe_in, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&P->pipe_out, cudaStreamNonBlocking);
+        if (e != cudaSuccess) return cuda_fail(e, "host pipeline streams");
+    }
+    while (int(P->pipe_ev.size()) < 2 + 2 * chunks) {
+        cudaEvent_t ev;
+        e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+        if (e != cudaSuccess) return cuda_fail(e, "host pipeline events");
+        P->pipe_ev.push_back(ev);
+    }
+    bool same = P->pipe_cols == cols && P->pipe_chunks == chunks &&
+                int(P->pipe_xd.size()) == p && int(P->pipe_yd.size()) == p;
+    for (int i = 0; i < p && same; i++) same = P->pipe_xd[i] == x_dev[i] && P->pipe_yd[i] == y_dev[i];
+    if (same) return DPDR_OK;
+    const size_t bytes = sizeof(void*) * 2 * size_t(p) * chunks;
+    if (bytes > P->d_pipe_bytes) {
+        if (P->d_pipe) cudaFree(P->d_pipe);
+        P->d_pipe = nullptr;
+        P->d_pipe_bytes = 0;
+        e = cudaMalloc(&P->d_pipe, bytes);
+        if (e != cudaSuccess) return cuda_fail(e, "host pipeline tables");
+        P->d_pipe_bytes = bytes;
+    }
+    std::vector<const char*> t(2 * size_t(p) * chunks);
+    for (int c = 0; c < chunks; c++)
+        for (int i = 0; i < p; i++) {
+            t[(size_t(c) * 2) * p + i] = static_cast<const char*>(x_dev[i]) + c * cols * es;
+            t[(size_t(c) * 2 + 1) * p + i] = static_cast<const char*>(y_dev[i]) + c * cols * es;
+        }
+    e = cudaMemcpy(P->d_pipe, t.data(), bytes, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "host pipeline table upload");
+    P->pipe_cols = cols;
+    P->pipe_chunks = chunks;
+    P->pipe_xd.assign(x_dev, x_dev + p);
+    P->pipe_yd.assign(y_dev, y_dev + p);
+    (void)vec;
+    return DPDR_OK;
+}
+
 extern "C" int dpdr_allreduce_host(dpdr_plan_t h, const void* const* x_host,
                                    void* const* y_host, void* const* x_dev,
                                    void* const* y_dev, dpdr_stream_t stream)
@@ -133,20 +186,48 @@ extern "C" int dpdr_allreduce_host(dpdr_plan_t h, const void* const* x_host,
     if (!x_host || !y_host || !x_dev || !y_dev)
         return fail(DPDR_ERR_INVALID, "dpdr_allreduce_host: NULL pointer array");
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    const size_t bytes = size_t(P->m) * P->esize;
     for (int i = 0; i < P->p; i++)
         if (!x_host[i] || !y_host[i]) return fail(DPDR_ERR_INVALID, "NULL host buffer");
-    cudaError_t e;
-    for (int i = 0; i < P->p && bytes; i++) {
-        e = cudaMemcpyAsync(x_dev[i], x_host[i], bytes, cudaMemcpyHostToDevice, s);
-        if (e != cudaSuccess) return cuda_fail(e, "host to device copy");
-    }
-    int rc = dpdr_allreduce(h, reinterpret_cast<const void* const*>(x_dev), y_dev, stream);
+    if (P->m == 0) return DPDR_OK;
+    int vec = 0;
+    int rc = check_buffers(P, reinterpret_cast<const void* const*>(x_dev),
+                           reinterpret_cast<const void* const*>(y_dev), &vec);
     if (rc) return rc;
-    for (int i = 0; i < P->p && bytes; i++) {
-        e = cudaMemcpyAsync(y_host[i], y_dev[i], bytes, cudaMemcpyDeviceToHost, s);
+    rc = pipe_prepare(P, x_dev, y_dev, vec != 0);
+    if (rc) return rc;
+    const int p = P->p, C = P->pipe_chunks;
+    const int64_t es = int64_t(P->esize);
+    cudaEvent_t entry = P->pipe_ev[0], done = P->pipe_ev[1];
+    cudaError_t e = cudaEventRecord(entry, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(P->pipe_in, entry, 0);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(P->pipe_out, entry, 0);
+    if (e != cudaSuccess) return cuda_fail(e, "host pipeline entry");
+    char* const* tab = reinterpret_cast<char* const*>(P->d_pipe);
+    for (int c = 0; c < C; c++) {
+        const int64_t c0 = c * P->pipe_cols, mc = std::min<int64_t>(P->pipe_cols, P->m - c0);
+        const size_t off = size_t(c0 * es), len = size_t(mc * es);
+        cudaEvent_t in = P->pipe_ev[2 + 2 * c], out = P->pipe_ev[3 + 2 * c];
+        for (int i = 0; i < p && e == cudaSuccess; i++)
+            e = cudaMemcpyAsync(static_cast<char*>(x_dev[i]) + off,
+                                static_cast<const char*>(x_host[i]) + off, len,
+                                cudaMemcpyHostToDevice, P->pipe_in);
+        if (e == cudaSuccess) e = cudaEventRecord(in, P->pipe_in);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(s, in, 0);
+        if (e != cudaSuccess) return cuda_fail(e, "host to device copy");
+        rc = fused_launch_cols(P, reinterpret_cast<const char* const*>(tab + size_t(c) * 2 * p),
+                               tab + (size_t(c) * 2 + 1) * p, mc, vec != 0, s);
+        if (rc) return rc;
+        e = cudaEventRecord(out, s);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(P->pipe_out, out, 0);
+        for (int i = 0; i < p && e == cudaSuccess; i++)
+            e = cudaMemcpyAsync(static_cast<char*>(y_host[i]) + off,
+                                static_cast<const char*>(y_dev[i]) + off, len,
+                                cudaMemcpyDeviceToHost, P->pipe_out);
         if (e != cudaSuccess) return cuda_fail(e, "device to host copy");
     }
+    e = cudaEventRecord(done, P->pipe_out);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, done, 0);
+    if (e != cudaSuccess) return cuda_fail(e, "host pipeline exit");
     return DPDR_OK;
 }
 

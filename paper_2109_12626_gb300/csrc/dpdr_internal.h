@@ -54,6 +54,7 @@ struct Plan {
     int sched_rpc = 0;         // ranks per CTA, 0 = auto
     int sched_slices = 0;      // CTAs per rank (column slices), 0 = auto
     int split_depth = -1;      // cut depth of the split layout, -1 = auto
+    int64_t host_chunk = int64_t(1) << 30;  // bytes of rank data per host-pipeline chunk
 
     // device memory: one allocation carved into the tables below
     char* dmem = nullptr;
@@ -92,6 +93,17 @@ struct Plan {
     char* d_part = nullptr;
     int64_t part_stride = 0;
 
+    // host-buffer pipeline of dpdr_allreduce_host (api.cpp), made on first use:
+    // column chunks copied in on one stream, reduced on the caller's stream,
+    // copied out on another
+    cudaStream_t pipe_in = nullptr, pipe_out = nullptr;
+    std::vector<cudaEvent_t> pipe_ev;            // entry, done, then in/out per chunk
+    char* d_pipe = nullptr;                      // per-chunk rank-pointer tables
+    size_t d_pipe_bytes = 0;
+    int64_t pipe_cols = 0;
+    int pipe_chunks = 0;
+    std::vector<const void*> pipe_xd, pipe_yd;
+
     // facts
     int last_vector_path = 0;
     int sched_ctas = 0, sched_ranks_per_cta = 0;
@@ -116,6 +128,8 @@ int stage_pointers(Plan* P, const void* const* x, const void* const* y,
 
 // launchers
 int fused_launch(Plan* P, cudaStream_t s);      // fused.cu
+int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t mc, bool vec,
+                      cudaStream_t s);             // fused.cu
 int fused_auto_mode(const Plan* P);             // fused.cu
 int fused_split_prepare(Plan* P, bool force, int depth);  // fused.cu
 int schedule_launch(Plan* P, cudaStream_t s);   // schedule.cu

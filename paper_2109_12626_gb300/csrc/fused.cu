@@ -545,15 +545,23 @@ int fused_split_prepare(Plan* P, bool force, int depth)
 
 int fused_launch(Plan* P, cudaStream_t s)
 {
-    if (P->m == 0) return DPDR_OK;
+    return fused_launch_cols(P, P->d_x, P->d_y, P->m, P->last_vector_path != 0, s);
+}
+
+// The fused kernel on mc columns, with device tables of rank pointers that
+// may point into the middle of the rank buffers (a column chunk).
+int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t mc, bool vec,
+                      cudaStream_t s)
+{
+    if (mc == 0) return DPDR_OK;
     int mode = P->fused_mode ? P->fused_mode : fused_auto_mode(P);
     const int lg = tile_lg_wu(P);
     if (mode == 2 && lg < 0) return fail(DPDR_ERR_INVALID, "tile mode: p too large");
     if (mode == 3 && !P->split_ready) return fail(DPDR_ERR_INVALID, "split mode: p < 2");
 
     FusedArgs a;
-    a.x = P->d_x;
-    a.y = P->d_y;
+    a.x = dx;
+    a.y = dy;
     a.tape = P->d_tape;
     a.levels = P->d_levels;
     a.level_off = P->d_level_off;
@@ -561,11 +569,10 @@ int fused_launch(Plan* P, cudaStream_t s)
     a.p = P->p;
     a.r0 = P->r0;
     a.r1 = P->r1;
-    const bool vec = P->last_vector_path != 0;
     const int epv = int(16 / P->esize);
-    a.nvec = vec ? P->m / epv : 0;
+    a.nvec = vec ? mc / epv : 0;
     a.scalar_base = a.nvec * epv;
-    a.nscalar = P->m - a.scalar_base;
+    a.nscalar = mc - a.scalar_base;
     a.lg_wu = lg < 0 ? 0 : lg;
     a.vec_tiles = (a.nvec + (int64_t(1) << a.lg_wu) - 1) >> a.lg_wu;
     a.seg = P->d_seg;

@@ -209,6 +209,10 @@ static void free_plan(Plan* P)
 {
     if (!P) return;
     if (P->staged) cudaEventDestroy(P->staged);
+    for (cudaEvent_t e : P->pipe_ev) cudaEventDestroy(e);
+    if (P->pipe_in) cudaStreamDestroy(P->pipe_in);
+    if (P->pipe_out) cudaStreamDestroy(P->pipe_out);
+    if (P->d_pipe) cudaFree(P->d_pipe);
     if (P->d_split) cudaFree(P->d_split);
     if (P->d_sched) cudaFree(P->d_sched);
     if (P->h_ptrs) cudaFreeHost(P->h_ptrs);
@@ -387,6 +391,10 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
         P->split_depth = int(v);
         return fused_split_prepare(P, true, P->split_depth);
     }
+    case DPDR_OPT_HOST_CHUNK_BYTES:
+        if (v < 4096) return fail(DPDR_ERR_INVALID, "host chunk below 4096 bytes");
+        P->host_chunk = v;
+        return DPDR_OK;
     case DPDR_OPT_BLOCKS: {
         if (v < 0) return fail(DPDR_ERR_INVALID, "b < 0");
         const int nb = clamp_b(P->m, v == 0 ? block_count_rule(P->p, P->m, 0) : v);

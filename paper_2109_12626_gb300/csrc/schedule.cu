@@ -119,8 +119,10 @@ __device__ __forceinline__ bool cta_wait(const SchedArgs& a, const uint32_t* ctr
     if (threadIdx.x == 0) {
         int r = 1;
         if (ld_acquire(ctr) < target) {
+            // poll hot first (a partner is usually a few hundred ns away),
+            // then back off gently; every poll checks the time bound
             const uint64_t t0 = now_ns();
-            unsigned sleep = 32;
+            unsigned sleep = 0, polls = 0;
             while (true) {
                 if (ld_acquire(ctr) >= target) break;
                 if (ld_relaxed(a.abort_flag)) { r = 0; break; }
@@ -135,8 +137,10 @@ __device__ __forceinline__ bool cta_wait(const SchedArgs& a, const uint32_t* ctr
                     r = 0;
                     break;
                 }
-                __nanosleep(sleep);
-                if (sleep < 1024) sleep <<= 1;
+                if (++polls > 32) {
+                    sleep = sleep ? (sleep < 256 ? sleep * 2 : 256) : 32;
+                    __nanosleep(sleep);
+                }
             }
         }
         ok = r;

@@ -187,19 +187,28 @@ def test_repeated_calls_and_pointer_changes(pkg, orc):
                 _check_all(ys2, want)
 
 
-def test_host_buffers_end_to_end(pkg, orc):
-    kind, p, m = "float32", 32, 10007
-    x = host_inputs(kind, 31, p, m, sigma=1e-3)
+@pytest.mark.parametrize("kind,p,m,chunk", [("float32", 32, 10007, 0), ("float32", 32, 10007, 4096),
+                                            ("int32", 1152, 3001, 65536), ("mat2x2u32", 7, 2049, 4096),
+                                            ("float32", 3, 257, 4096)])
+@pytest.mark.parametrize("in_place", [False, True])
+def test_host_buffers_end_to_end(pkg, orc, kind, p, m, chunk, in_place):
+    """dpdr_allreduce_host: pinned host inputs, column chunks pipelined
+    through copy-in, kernel and copy-out streams, pinned host outputs."""
+    x = host_inputs(kind, 31, p, m)
     want = _want(orc, x, kind)
     dev = torch.device("cuda:0")
-    xh = [torch.from_numpy(x[i].copy()).pin_memory() for i in range(p)]
-    yh = [torch.zeros(m).pin_memory() for _ in range(p)]
-    xd = [torch.empty(m, device=dev) for _ in range(p)]
-    yd = [torch.empty(m, device=dev) for _ in range(p)]
+    xh = [torch.from_numpy(np.ascontiguousarray(x[i]).view(np.int32).reshape(-1).copy()).pin_memory()
+          for i in range(p)]
+    yh = [torch.full_like(t, -9).pin_memory() for t in xh]
+    xd = [torch.empty_like(t, device=dev) for t in xh]
+    yd = xd if in_place else [torch.empty_like(t, device=dev) for t in xh]
     with pkg.Plan(p, m, kind, 0) as plan:
-        plan.allreduce_host(xh, yh, xd, yd)
-        plan.sync()
-    _check_all(yh, want)
+        if chunk:
+            plan.set(pkg.OPT_HOST_CHUNK_BYTES, chunk)
+        for _ in range(2):
+            plan.allreduce_host(xh, yh, xd, yd)
+            plan.sync()
+            _check_all(yh, want)
 
 
 def test_invalid_arguments(pkg):
