@@ -125,7 +125,7 @@ __device__ __forceinline__ bool cta_wait(const SchedArgs& a, const uint32_t* ctr
             unsigned sleep = 0, polls = 0;
             while (true) {
                 if (ld_acquire(ctr) >= target) break;
-                if (ld_relaxed(a.abort_flag)) { r = 0; break; }
+                if ((polls & 15) == 15 && ld_relaxed(a.abort_flag)) { r = 0; break; }
                 if (now_ns() - t0 > uint64_t(a.wait_ns)) {
                     if (atomicCAS(a.err, 0u, uint32_t(DPDR_ERR_TIMEOUT)) == 0u) {
                         a.err[1] = uint32_t(rank);
@@ -151,14 +151,14 @@ __device__ __forceinline__ bool cta_wait(const SchedArgs& a, const uint32_t* ctr
     return r != 0;
 }
 
-// Release the CTA's writes to the rank's partner(s).
+// Release the CTA's writes to the rank's partner(s): the barrier orders
+// every thread's block writes before thread 0's gpu-scope release store
+// (release is cumulative over what thread 0 has observed), and the partner's
+// acquire load orders its reads after it.
 __device__ __forceinline__ void publish(const SchedArgs& a, uint32_t* ctr, uint32_t v, int rank)
 {
     __syncthreads();
-    if (threadIdx.x == 0 && rank != a.skip_rank) {
-        __threadfence();
-        st_release(ctr, v);
-    }
+    if (threadIdx.x == 0 && rank != a.skip_rank) st_release(ctr, v);
 }
 
 // dst[k] = lo[k] (.) hi[k] for k in [s, e); rows are virtual bases indexed
