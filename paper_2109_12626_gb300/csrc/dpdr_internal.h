@@ -47,7 +47,7 @@ struct Plan {
     std::vector<int> level_off;                // nlevels + 1
 
     // options
-    int fused_mode = 0;        // 0 auto, 1 stream, 2 tile
+    int fused_mode = 0;        // 0 auto, 1 stream, 2 tile, 3 split, 4 bulk
     int64_t wait_ns = 4000000000LL;
     int skip_rank = -1;
     int sched_threads = 128;
@@ -81,7 +81,7 @@ struct Plan {
 
     // dynamic shared memory already granted to the fused kernels of this
     // plan's element type (stream, tile), so launches skip the attribute call
-    int smem_attr[3] = {48 * 1024, 48 * 1024, 48 * 1024};
+    int smem_attr[4] = {48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024};
 
     // split layout of the fused kernel (fused.cu): subtrees at depth split_s
     bool split_ready = false;

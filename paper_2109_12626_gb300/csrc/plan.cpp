@@ -357,7 +357,7 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
     if (!P) return fail(DPDR_ERR_INVALID, "dpdr_plan_set: NULL plan");
     switch (key) {
     case DPDR_OPT_FUSED_MODE:
-        if (v < 0 || v > 3) return fail(DPDR_ERR_INVALID, "fused mode: 0, 1, 2 or 3");
+        if (v < 0 || v > 4) return fail(DPDR_ERR_INVALID, "fused mode: 0 to 4");
         if (v == 3) {
             int rc = fused_split_prepare(P, true, P->split_depth);
             if (rc) return rc;

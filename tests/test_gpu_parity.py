@@ -56,7 +56,7 @@ def _check_all(ys, want, guards=None):
 
 
 @pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
-@pytest.mark.parametrize("mode", [1, 2, 3], ids=["stream", "tile", "split"])
+@pytest.mark.parametrize("mode", [1, 2, 3, 4], ids=["stream", "tile", "split", "bulk"])
 def test_fused_matches_oracle(pkg, orc, case, mode):
     _, kind, seed, p, m, kw, _ = case
     dev = torch.device("cuda:0")
@@ -93,7 +93,7 @@ def test_schedule_matches_oracle(pkg, orc, case):
         assert np.array_equal(bits(xs[i]), expect_bits(x[i]))
 
 
-FUSED_RUNS = {"fused_stream": 1, "fused_tile": 2, "fused_split": 3}
+FUSED_RUNS = {"fused_stream": 1, "fused_tile": 2, "fused_split": 3, "fused_bulk": 4}
 RUNS = list(FUSED_RUNS) + ["schedule"]
 
 
