@@ -47,7 +47,13 @@ DEFAULT_WORKLOAD = "p32_m134217728_f32"
 METRIC = "allreduce GB/s (p*m*sizeof read + p*m*sizeof written)"
 ESIZE = {"int32": 4, "float32": 4, "mat2x2u32": 16}
 DTYPE_TAG = {"int32": "int32", "float32": "f32", "mat2x2u32": "u32"}
-KERNEL_SOURCES = {"fused": "fused.cu", "schedule": "schedule.cu"}
+# source files whose change invalidates a layout's measured DRAM traffic
+KERNEL_SOURCES = {"stream": ("fused_stream.cu", "fused_common.cuh"),
+                  "tile": ("fused_tile.cu", "fused_common.cuh"),
+                  "split": ("fused_split.cu", "fused_common.cuh"),
+                  "bulk": ("fused_bulk.cu", "fused_common.cuh"),
+                  "schedule": ("schedule.cu",)}
+LAYOUTS = {1: "stream", 2: "tile", 3: "split", 4: "bulk"}
 
 
 # ------------------------------------------------------------ workload
@@ -167,7 +173,7 @@ def measured_peak_gbs() -> tuple[float, str]:
 
 def kernel_source_hash(kernel: str) -> str:
     h = hashlib.sha256()
-    for f in (KERNEL_SOURCES[kernel], "ops.cuh"):
+    for f in KERNEL_SOURCES[kernel] + ("ops.cuh",):
         with open(os.path.join(ROOT, "paper_2109_12626_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -341,7 +347,6 @@ def main(argv=None) -> int:
     achieved = algo_bytes / (avg_launch * 1e-3) / 1e9
     peak, peak_kind = measured_peak_gbs()
     units = p * m
-    traffic = profiled_traffic(args.kernel, args.workload, units)
 
     # end to end with host buffers
     e2e = None
@@ -375,7 +380,8 @@ def main(argv=None) -> int:
                "sample": sample}
 
     info = plan.info()
-    launches_per_step = 2 if (args.kernel == "fused" and (args.mode or info["auto_mode"]) == 3) else 1
+    layout = LAYOUTS[args.mode or info["auto_mode"]] if args.kernel == "fused" else "schedule"
+    launches_per_step = 2 if layout == "split" else 1
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
@@ -390,10 +396,10 @@ def main(argv=None) -> int:
                    "l2": "inputs larger than L2 (%.1f GB), no flush" % (algo_bytes / 2e9)
                    if algo_bytes / 2 > 129e6 else "working set fits L2: warm-cache number",
                    "parallelism": "replicas" if world > 1 else "single GPU"},
-        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+        "roofline": {"bound": "hbm", "kernel": layout, "achieved": round(achieved, 1), "peak": peak,
                      "unit": "GB/s", "frac": round(achieved / peak, 4),
                      "peak_kind": peak_kind + " copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
-                     "traffic": traffic,
+                     "traffic": profiled_traffic(layout, args.workload, units),
                      "kernel_ms": round(avg_launch, 4)},
         "cpu_baseline": cpu,
         "e2e": e2e,

@@ -26,7 +26,7 @@
  * bottom = (-1,-1).  The witness is associative and non-commutative and fails
  * on any misordered, dropped or repeated operand.
  *
- * Readings of the paper this file takes (all listed in the design doc):
+ * Readings of the paper this file takes:
  *   - d_i is the DEPTH of processor i (the correctness argument of Sec. 1.1
  *     uses depth; the caption of Algorithm 1 says height).
  *   - tree 0 = ranks [0, floor(p/2)), tree 1 = [floor(p/2), p), both
