@@ -81,7 +81,7 @@ struct Plan {
 
     // dynamic shared memory already granted to the fused kernels of this
     // plan's element type (stream, tile), so launches skip the attribute call
-    int smem_attr[5] = {48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024};
+    int smem_attr[4] = {48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024};
 
     // split layout of the fused kernel (fused.cu): subtrees at depth split_s
     bool split_ready = false;

@@ -149,7 +149,6 @@ int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t m
     a.group = P->split_group;
     a.bulk_tiles = vec ? (a.nvec * 16) / kBulkTile : 0;
     a.bulk_bar_off = 0;
-    a.unit_base = 0;
     a.err = P->d_err;
     a.wait_ns = P->wait_ns;
     if (mode == 4 && !vec) mode = 1;  // bulk copies need 16-byte aligned rows

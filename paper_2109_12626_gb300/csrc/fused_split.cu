@@ -48,10 +48,9 @@ __device__ __forceinline__ void split_reduce_column(const FusedArgs& a, int g, i
     U::st_keep(row, u, acc);
 }
 
-// the top-of-tree fold of one column: y = v(r0) (.) v(r1)
 template <class U>
-__device__ __forceinline__ typename U::T split_finish_fold(const FusedArgs& a, int64_t u,
-                                                           typename U::T* slot, int stride)
+__device__ __forceinline__ void split_finish_column(const FusedArgs& a, int r, int64_t u,
+                                                    typename U::T* slot, int stride)
 {
     using T = typename U::T;
     const int n = a.nitems;
@@ -77,14 +76,7 @@ __device__ __forceinline__ typename U::T split_finish_fold(const FusedArgs& a, i
 #pragma unroll
         for (int k = 0; k < kStreamAhead; k++) cur[k] = nxt[k];
     }
-    return (a.p >= 2) ? U::op(slot[0], acc) : acc;
-}
-
-template <class U>
-__device__ __forceinline__ void split_finish_column(const FusedArgs& a, int r, int64_t u,
-                                                    typename U::T* slot, int stride)
-{
-    const typename U::T y = split_finish_fold<U>(a, u, slot, stride);
+    const T y = (a.p >= 2) ? U::op(slot[0], acc) : acc;
     const int i1 = min(a.p, (r + 1) * a.group);
 #pragma unroll 4
     for (int i = r * a.group; i < i1; i++) U::st(rank_ptr_w(a.y, i), u, y);
@@ -110,7 +102,7 @@ __global__ void __launch_bounds__(kStreamThreads, 3)
 fused_split_finish_kernel(FusedArgs a)
 {
     extern __shared__ uint4 smem[];
-    const int64_t u = a.unit_base + int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+    const int64_t u = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
     if (u < a.nvec) {
         split_finish_column<VecUnit<Op>>(a, blockIdx.y, u, smem + threadIdx.x, blockDim.x);
     } else if (u < a.nvec + a.nscalar) {
@@ -120,30 +112,6 @@ fused_split_finish_kernel(FusedArgs a)
     }
 }
 
-// Finish kernel for whole 4 KB column tiles: the CTA folds its 256 columns,
-// puts the result tile in shared memory, and its first warp hands the
-// group's rank outputs to the TMA unit as bulk stores of that one tile, so
-// the write phase does not queue p 16-byte stores per thread.
-template <class Op>
-__global__ void __launch_bounds__(kStreamThreads, 3)
-fused_split_finish_bulk_kernel(FusedArgs a)
-{
-    extern __shared__ uint4 smem[];
-    const int tid = threadIdx.x;
-    uint4* tile = smem + int64_t(a.bulk_bar_off) * kStreamThreads;  // after the slots
-    const int64_t t = blockIdx.x;
-    tile[tid] = split_finish_fold<VecUnit<Op>>(a, t * kStreamThreads + tid, smem + tid, kStreamThreads);
-    fence_async_shared();
-    __syncthreads();
-    if (tid < 32) {
-        const int r = blockIdx.y;
-        const int i1 = min(a.p, (r + 1) * a.group);
-        for (int i = r * a.group + tid; i < i1; i += 32)
-            bulk_store(rank_ptr_w(a.y, i) + t * (kStreamThreads * 16), tile, kStreamThreads * 16);
-        bulk_commit();
-        bulk_wait_read_all();  // the tile must stay in shared memory until read
-    }
-}
 
 template <class Op>
 struct Split {
@@ -166,29 +134,8 @@ struct Split {
         const int groups = (P->p + a.group - 1) / a.group;
         fused_split_reduce_kernel<Op>
             <<<dim3(unsigned(blocks), unsigned(P->split_nseg)), kStreamThreads, smem, s>>>(a);
-        // whole 4 KB tiles of 16-byte units go through bulk stores, the rest
-        // (a partial tile, single elements) through the plain finish kernel
-        const int64_t tiles = a.nvec / kStreamThreads;
-        if (tiles > 0) {
-            const size_t smem_b = smem + kStreamThreads * sizeof(uint4);
-            if (int(smem_b) > P->smem_attr[4]) {
-                cudaError_t e = cudaFuncSetAttribute(fused_split_finish_bulk_kernel<Op>,
-                                                     cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                     int(smem_b));
-                if (e != cudaSuccess) return cuda_fail(e, "fused split attribute");
-                P->smem_attr[4] = int(smem_b);
-            }
-            FusedArgs b = a;
-            b.bulk_bar_off = P->max_depth + 1;  // slot rows before the tile
-            fused_split_finish_bulk_kernel<Op>
-                <<<dim3(unsigned(tiles), unsigned(groups)), kStreamThreads, smem_b, s>>>(b);
-        }
-        a.unit_base = tiles * kStreamThreads;
-        const int64_t rest = units - a.unit_base;
-        if (rest > 0)
-            fused_split_finish_kernel<Op>
-                <<<dim3(unsigned((rest + kStreamThreads - 1) / kStreamThreads), unsigned(groups)),
-                   kStreamThreads, smem, s>>>(a);
+        fused_split_finish_kernel<Op>
+            <<<dim3(unsigned(blocks), unsigned(groups)), kStreamThreads, smem, s>>>(a);
         return launched();
     }
 };
