@@ -259,6 +259,117 @@ def run_reference(args, w) -> dict:
                     "d2h_bytes_per_step": 0}}
 
 
+# -------------------------------------------------------------- sweeps
+def model_rounds(p: int) -> int:
+    """Unit steps before the first block reaches the last leaf in the
+    schedule's rendezvous model (4h-7 for p = 2^h - 2, h >= 3)."""
+    h = 0
+    while (1 << h) < p + 2:
+        h += 1
+    return max(1, 4 * h - 7)
+
+
+def fit_cost_model(p: int, m: int, points):
+    """Least-squares fit of T(b) = T0 + (L + 3(b-1)) (alpha + beta m / b)
+    (Sec. 1.2's cost model plus a launch constant T0) to (b, seconds)
+    points; returns T0, alpha, beta (seconds, seconds/element)."""
+    import numpy as np
+    L = model_rounds(p)
+    A = np.array([[1.0, L + 3 * (b - 1), (L + 3 * (b - 1)) * m / b] for b, _ in points])
+    y = np.array([t for _, t in points])
+    coef, *_ = np.linalg.lstsq(A, y, rcond=None)
+    return float(coef[0]), float(coef[1]), float(coef[2])
+
+
+def _timed(fn, reps, stream, graph=False):
+    import torch
+    for _ in range(2):
+        fn()
+    torch.cuda.synchronize()
+    g = None
+    if graph:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for _ in range(reps):
+                fn()
+        g.replay()
+        torch.cuda.synchronize()
+    a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    if g is not None:
+        g.replay()
+    else:
+        for _ in range(reps):
+            fn()
+    z.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(z) / reps * 1e-3
+
+
+def run_sweep(args, w) -> int:
+    """--sweep m: every m = 2^0 .. 2^k of the workload, fused kernel (its
+    automatic layout, CUDA-graph replay so launch overhead is excluded) and
+    schedule kernel at the block-count rule.  --sweep b: the schedule
+    kernel's time against b at one m, with the Sec. 1.2 cost model fitted.
+    One JSON line per point, then a summary line."""
+    import torch
+    import paper_2109_12626_gb300 as pkg
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    p, kind, es = w["p"], w["kind"], ESIZE[w["kind"]]
+    if args.sweep == "m":
+        top = int(args.m or (1 << 23)).bit_length() - 1
+        for k in range(0, top + 1):
+            m = 1 << k
+            ww = dict(w, m=m)
+            xs = gen_device_inputs(ww, dev)
+            ys = [torch.empty_like(x) for x in xs]
+            rec = {"sweep": "m", "workload": args.workload, "p": p, "m": m}
+            with pkg.Plan(p, m, kind, 0) as plan:
+                bd = plan.bind(xs, ys)
+                t = _timed(lambda: bd.allreduce(), 20, None, graph=True)
+                info = plan.info()
+                rec["fused"] = {"us": round(t * 1e6, 2), "gbs": round(2 * p * m * es / t / 1e9, 2),
+                                "layout": LAYOUTS[info["auto_mode"]],
+                                "split_depth": info["split_depth"] if info["auto_mode"] == 3 else None}
+                t = _timed(lambda: bd.allreduce_schedule(), 3 if m >= (1 << 20) else 10, None)
+                plan.sync()
+                rec["schedule"] = {"b": info["b"], "us": round(t * 1e6, 2),
+                                   "gbs": round(2 * p * m * es / t / 1e9, 2),
+                                   "slices": plan.info()["sched_slices"]}
+            print(json.dumps(rec), flush=True)
+            del xs, ys
+            torch.cuda.empty_cache()
+        return 0
+    # --sweep b
+    m = w["m"]
+    xs = gen_device_inputs(w, dev)
+    ys = [torch.empty_like(x) for x in xs]
+    bs = sorted(set(int(v) for v in args.blist.split(",") if int(v) <= max(m, 1)))
+    points = []
+    for b in bs:
+        with pkg.Plan(p, m, kind, b) as plan:
+            bd = plan.bind(xs, ys)
+            t = _timed(lambda: bd.allreduce_schedule(), 5 if m >= (1 << 20) else 10, None)
+            plan.sync()
+            points.append((b, t))
+            print(json.dumps({"sweep": "b", "workload": args.workload, "p": p, "m": m, "b": b,
+                              "us": round(t * 1e6, 2), "slices": plan.info()["sched_slices"]}),
+                  flush=True)
+    t0, alpha, beta = fit_cost_model(p, m, points)
+    best = min(points, key=lambda x: x[1])
+    kappa = alpha / beta if beta > 0 else float("inf")
+    rule = pkg.block_count_rule(p, m, kappa) if beta > 0 and alpha > 0 else None
+    print(json.dumps({"sweep": "b-fit", "workload": args.workload, "p": p, "m": m,
+                      "rounds_L": model_rounds(p), "T0_us": round(t0 * 1e6, 3),
+                      "alpha_us": round(alpha * 1e6, 4), "beta_ns_per_elem": round(beta * 1e9, 5),
+                      "kappa_elems": round(kappa, 1) if beta > 0 else None,
+                      "best_b": best[0], "best_us": round(best[1] * 1e6, 2),
+                      "rule_b_with_fitted_kappa": rule,
+                      "rule_b_default_kappa": pkg.block_count_rule(p, m)}), flush=True)
+    return 0
+
+
 # ---------------------------------------------------------------- main
 def main(argv=None) -> int:
     ap = argparse.ArgumentParser()
@@ -275,6 +386,9 @@ def main(argv=None) -> int:
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--sweep", choices=("m", "b"), default=None,
+                    help="m: all m = 2^k up to --m; b: schedule time against b")
+    ap.add_argument("--blist", default="1,2,4,8,16,32,64,128,256,512,1024")
     args = ap.parse_args(argv)
     args.warmup = max(args.warmup, 3)
 
@@ -285,6 +399,8 @@ def main(argv=None) -> int:
         if rank == 0:
             print(json.dumps(run_reference(args, w)), flush=True)
         return 0
+    if args.sweep:
+        return run_sweep(args, w)
 
     import torch
     import paper_2109_12626_gb300 as pkg

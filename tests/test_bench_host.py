@@ -88,3 +88,25 @@ def test_reference_arm_prints_one_json_line():
     assert d["impl"] == "reference" and d["unit"] == "GB/s" and d["value"] > 0
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] == 1
     assert d["e2e"]["h2d_bytes_per_step"] == 0
+
+
+def test_cost_model_fit_recovers_known_constants():
+    """The Sec. 1.2 model T(b) = T0 + (L + 3(b-1))(alpha + beta m / b) fitted
+    to exact model points returns the constants it was made from, and the
+    block-count rule with the fitted kappa = alpha/beta lands on the model's
+    best b."""
+    p, m = 1152, 1 << 22
+    T0, alpha, beta = 8e-6, 2.5e-6, 0.4e-9
+    L = bench.model_rounds(p)
+    assert L == 4 * 11 - 7
+    pts = [(b, T0 + (L + 3 * (b - 1)) * (alpha + beta * m / b)) for b in (1, 4, 16, 64, 256, 1024)]
+    t0, a, bta = bench.fit_cost_model(p, m, pts)
+    assert t0 == pytest.approx(T0, rel=1e-6) and a == pytest.approx(alpha, rel=1e-6)
+    assert bta == pytest.approx(beta, rel=1e-6)
+    import math
+    T = lambda b: T0 + (L + 3 * (b - 1)) * (alpha + beta * m / b)
+    best = min(range(1, 5000), key=T)
+    kappa = a / bta
+    h = 11
+    rule = round(math.sqrt((4 * h - 6) * m / (3 * kappa)))
+    assert T(rule) <= T(best) * 1.01
