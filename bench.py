@@ -277,7 +277,14 @@ def fit_cost_model(p: int, m: int, points):
     L = model_rounds(p)
     A = np.array([[1.0, L + 3 * (b - 1), (L + 3 * (b - 1)) * m / b] for b, _ in points])
     y = np.array([t for _, t in points])
-    coef, *_ = np.linalg.lstsq(A, y, rcond=None)
+    try:  # the constants are times: fit them non-negative
+        from scipy.optimize import nnls
+        scale = A.max(axis=0)
+        scale[scale == 0] = 1.0
+        coef, _ = nnls(A / scale, y)
+        coef = coef / scale
+    except ImportError:
+        coef, *_ = np.linalg.lstsq(A, y, rcond=None)
     return float(coef[0]), float(coef[1]), float(coef[2])
 
 

@@ -17,13 +17,14 @@ static int64_t stream_target(const Plan* P) { return int64_t(P->num_sms) * 1024;
 //    whose read phase (first kernel) and write phase (second kernel) keep
 //    HBM traffic one-directional; it beats column streaming from m = 2^15 up
 //    to the largest sizes at p = 1152;
-//  * otherwise column streaming once there are enough columns to fill the
-//    GPU, and the shared-memory tile below that.
+//  * otherwise column streaming once there are a quarter of the columns it
+//    needs to fill the GPU (p = 36, 2x2 matrices, m = 2^16: 13 us against the
+//    tile's 15 us), and the shared-memory tile below that.
 int fused_auto_mode(const Plan* P)
 {
     const int64_t units = P->m * int64_t(P->esize) / 16;
     if (P->p >= 128 && units >= 8192 && P->split_ready) return 3;
-    if (units >= stream_target(P)) return 1;
+    if (units >= stream_target(P) / 4) return 1;
     if (tile_lg_wu(P) >= 0) return 2;
     return P->split_ready ? 3 : 1;
 }
