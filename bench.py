@@ -162,6 +162,40 @@ def summarize_clocks(csv_text: str) -> dict | None:
             "reasons": sorted(reasons), "samples": len(load)}
 
 
+# ---------------------------------------------------------- host NUMA
+def gpu_local_cpus(dev_index: int):
+    """CPUs of the NUMA node the GPU is attached to (from sysfs), or None."""
+    import torch
+    try:
+        bus = torch.cuda.get_device_properties(dev_index).pci_bus_id  # "0000:01:00.0" on new torch
+    except Exception:
+        bus = None
+    if not bus:
+        try:
+            out = subprocess.run(["nvidia-smi", "-i", str(dev_index), "--query-gpu=pci.bus_id",
+                                  "--format=csv,noheader"], capture_output=True, text=True,
+                                 timeout=20).stdout.strip()
+            bus = out.splitlines()[0] if out else None
+        except (OSError, subprocess.SubprocessError):
+            bus = None
+    if not bus:
+        return None, None
+    bus = bus.lower()
+    if bus.count(":") == 2 and len(bus.split(":")[0]) == 8:
+        bus = bus[4:]  # nvidia-smi prints an 8-digit domain
+    try:
+        node = int(open("/sys/bus/pci/devices/%s/numa_node" % bus).read().strip())
+        if node < 0:
+            return None, None
+        cpus = set()
+        for part in open("/sys/devices/system/node/node%d/cpulist" % node).read().strip().split(","):
+            a, _, b = part.partition("-")
+            cpus.update(range(int(a), int(b or a) + 1))
+        return node, cpus or None
+    except (OSError, ValueError):
+        return None, None
+
+
 # ------------------------------------------------------------ roofline
 def measured_peak_gbs() -> tuple[float, str]:
     try:
@@ -474,10 +508,20 @@ def main(argv=None) -> int:
     # end to end with host buffers
     e2e = None
     if not args.no_e2e:
+        # pinned host buffers on the CPU node next to the GPU (first touch)
+        node, cpus = gpu_local_cpus(local)
+        saved = os.sched_getaffinity(0)
+        if cpus:
+            try:
+                os.sched_setaffinity(0, cpus)
+            except OSError:
+                node = None
         xh = [torch.empty(x.shape, dtype=x.dtype, pin_memory=True) for x in xs]
         yh = [torch.empty(x.shape, dtype=x.dtype, pin_memory=True) for x in xs]
         for h, x in zip(xh, xs):
             h.copy_(x)
+        for h in yh:
+            h.zero_()
         for _ in range(2):
             plan.allreduce_host(xh, yh, xs, ys, stream)
         plan.sync(stream)
@@ -493,8 +537,9 @@ def main(argv=None) -> int:
         t2 = max_over_ranks(s2.elapsed_time(e2), world, dev) / k2
         e2e = {"value": round(world * algo_bytes / (t2 * 1e-3) / 1e9, 3), "unit": "GB/s",
                "h2d_bytes_per_step": p * m * es, "d2h_bytes_per_step": p * m * es,
-               "steps": k2, "ms_per_step": round(t2, 3)}
+               "steps": k2, "ms_per_step": round(t2, 3), "host_numa_node": node}
         del xh, yh
+        os.sched_setaffinity(0, saved)
 
     cpu = None
     if rank == 0 and not args.no_cpu:
