@@ -185,10 +185,18 @@ static int build_tree(int lo, int n, int* parent, int* child0, int* child1,
     return ORC_OK;
 }
 
-int orc_trees(int p, int* parent, int* child0, int* child1, int* dual,
-              int* depth)
+/* topo 0: the dual trees of Sec. 1.1.  topo 1: one complete post-order tree
+ * over all p ranks, root p-1, no dual (the single doubly pipelined tree
+ * discussed in Sec. 1.2). */
+int orc_trees_topo(int p, int topo, int* parent, int* child0, int* child1,
+                   int* dual, int* depth)
 {
-    if (p < 1) return ORC_EINVAL;
+    if (p < 1 || topo < 0 || topo > 1) return ORC_EINVAL;
+    if (topo == 1) {
+        int rc = build_tree(0, p, parent, child0, child1, depth);
+        for (int i = 0; i < p; i++) dual[i] = -1;
+        return rc;
+    }
     int n0 = p / 2, n1 = p - n0;
     int rc = build_tree(0, n0, parent, child0, child1, depth);
     if (rc) return rc;
@@ -200,6 +208,12 @@ int orc_trees(int p, int* parent, int* child0, int* child1, int* dual,
         dual[p - 1] = n0 - 1;
     }
     return ORC_OK;
+}
+
+int orc_trees(int p, int* parent, int* child0, int* child1, int* dual,
+              int* depth)
+{
+    return orc_trees_topo(p, 0, parent, child0, child1, dual, depth);
 }
 
 /* ------------------------------------------------------------------ O3 ---
@@ -276,7 +290,9 @@ static int subtree_value(const foldctx* f, int i, char* out)
     return ORC_OK;
 }
 
-int orc_tree_fold(int p, int64_t m, int dt, const void* x, void* y)
+/* One tree (topo 1): y = v(p-1). */
+int orc_tree_fold_topo(int p, int topo, int64_t m, int dt, const void* x,
+                       void* y)
 {
     size_t s = esize(dt);
     if (p < 1 || m < 0 || s == 0) return ORC_EINVAL;
@@ -284,12 +300,12 @@ int orc_tree_fold(int p, int64_t m, int dt, const void* x, void* y)
     if (!T) return ORC_ENOMEM;
     int *par = T, *c0 = T + p, *c1 = T + 2 * p, *du = T + 3 * p,
         *dep = T + 4 * p;
-    int rc = orc_trees(p, par, c0, c1, du, dep);
+    int rc = orc_trees_topo(p, topo, par, c0, c1, du, dep);
     if (rc) { free(T); return rc; }
     foldctx f = {p, m, dt, s, (const char*)x, c0, c1};
-    int n0 = p / 2;
+    int n0 = topo == 1 ? 0 : p / 2;
     if (n0 == 0) {
-        rc = subtree_value(&f, p - 1, (char*)y); /* p == 1: y = x_0 */
+        rc = subtree_value(&f, p - 1, (char*)y); /* one root: y = v(p-1) */
     } else {
         size_t bytes = (size_t)m * s;
         char* v1 = (char*)malloc(bytes ? bytes : 1);
@@ -301,6 +317,11 @@ int orc_tree_fold(int p, int64_t m, int dt, const void* x, void* y)
     }
     free(T);
     return rc;
+}
+
+int orc_tree_fold(int p, int64_t m, int dt, const void* x, void* y)
+{
+    return orc_tree_fold_topo(p, 0, m, dt, x, y);
 }
 
 /* The full reduction-to-all contract on the CPU: the tree fold, then the
@@ -357,8 +378,8 @@ static int64_t blk_start(int64_t m, int b, int j)
 
 static int valid_blk(int b, int j) { return j >= 0 && j < b; }
 
-int orc_simulate(int p, int64_t m, int b, int dt, const void* x, void* y,
-                 int64_t* stats, int* last_round)
+int orc_simulate_topo(int p, int topo, int64_t m, int b, int dt,
+                      const void* x, void* y, int64_t* stats, int* last_round)
 {
     size_t s = esize(dt);
     if (p < 1 || m < 1 || b < 1 || b > m || s == 0) return ORC_EINVAL;
@@ -368,7 +389,7 @@ int orc_simulate(int p, int64_t m, int b, int dt, const void* x, void* y,
     if (!T) return ORC_ENOMEM;
     int *par = T, *c0 = T + p, *c1 = T + 2 * p, *du = T + 3 * p,
         *dep = T + 4 * p, *hgt = T + 5 * p;
-    rc = orc_trees(p, par, c0, c1, du, dep);
+    rc = orc_trees_topo(p, topo, par, c0, c1, du, dep);
     if (rc) { free(T); return rc; }
     /* node height, only for the planted mistake that confuses it with depth */
     for (int i = 0; i < p; i++) {
@@ -425,7 +446,10 @@ int orc_simulate(int p, int64_t m, int b, int dt, const void* x, void* y,
         arr0[i] = -1;
         ops_round_id[i] = -1;
     }
-    if (p == 1) arr0[0] = 0;
+    /* a root without a dual holds final block 0 once round 0's child
+     * exchanges are done; with no children at all, from the start */
+    for (int i = 0; i < p; i++)
+        if (par[i] < 0 && du[i] < 0 && c0[i] < 0) arr0[i] = 0;
 
     int64_t done_ops = 0, total_ops = 0, nex = 0;
     int64_t max_nonroot = 0, max_root = 0;
@@ -476,6 +500,9 @@ int orc_simulate(int p, int64_t m, int b, int dt, const void* x, void* y,
                     else
                         opv(dt, t, Yb, Yb, len); /* t (.) Y              */
                     if (o->kind == 3 && o->recv_blk == 0) arr0[me] = step;
+                    if (o->kind <= 1 && o->recv_blk == 0 && par[me] < 0 &&
+                        du[me] < 0)
+                        arr0[me] = step; /* lone root: block 0 final after its children */
                     if (ops_round_id[me] != o->round) {
                         ops_round_id[me] = o->round;
                         ops_round[me] = 0;
@@ -511,4 +538,10 @@ done:
     free(L); free(nops); free(cur); free(clk); free(arr0);
     free(sa); free(sb); free(ops_round); free(ops_round_id); free(T);
     return rc;
+}
+
+int orc_simulate(int p, int64_t m, int b, int dt, const void* x, void* y,
+                 int64_t* stats, int* last_round)
+{
+    return orc_simulate_topo(p, 0, m, b, dt, x, y, stats, last_round);
 }

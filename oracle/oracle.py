@@ -6,7 +6,8 @@ row-major ``[p][m]`` (``[p][m][4]`` uint32 words for 2x2 matrices,
 ``[p][m][2]`` int32 for the interval witness).
 
 Functions and the passages they follow:
-  trees(p)                 dual post-order trees, Sec. 1.1
+  trees(p, topo)           dual post-order trees, Sec. 1.1 (topo SINGLE: the
+                           one-tree variant of Sec. 1.2)
   left_fold(x, dt)         y = x_0 (.) ... (.) x_{p-1}, Sec. 1 problem statement
   tree_fold(x, dt)         post-order bracketing, Sec. 1.1 + Algorithm 1 roots
   allreduce(x, dt)         tree fold copied to all p rows
@@ -55,6 +56,12 @@ def lib():
         L = ctypes.CDLL(LIB_PATH)
         ip = ctypes.POINTER(ctypes.c_int)
         L.orc_trees.argtypes = [ctypes.c_int, ip, ip, ip, ip, ip]
+        L.orc_trees_topo.argtypes = [ctypes.c_int, ctypes.c_int, ip, ip, ip, ip, ip]
+        L.orc_tree_fold_topo.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int64,
+                                         ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p]
+        L.orc_simulate_topo.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int64,
+                                        ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+                                        ctypes.c_void_p, ctypes.POINTER(ctypes.c_int64), ip]
         for f in (L.orc_left_fold, L.orc_tree_fold, L.orc_allreduce):
             f.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_int,
                           ctypes.c_void_p, ctypes.c_void_p]
@@ -67,7 +74,8 @@ def lib():
                                         ctypes.c_void_p]
         L.orc_set_mutation.argtypes = [ctypes.c_int]
         for f in (L.orc_trees, L.orc_left_fold, L.orc_tree_fold,
-                  L.orc_allreduce, L.orc_simulate, L.orc_left_fold_f64):
+                  L.orc_allreduce, L.orc_simulate, L.orc_left_fold_f64,
+                  L.orc_trees_topo, L.orc_tree_fold_topo, L.orc_simulate_topo):
             f.restype = ctypes.c_int
         _lib = L
     return _lib
@@ -102,13 +110,16 @@ def set_mutation(k: int) -> None:
     lib().orc_set_mutation(int(k))
 
 
-def trees(p: int) -> dict:
+DUAL, SINGLE = 0, 1  # tree topologies: dual roots (Sec. 1.1), one tree (Sec. 1.2)
+
+
+def trees(p: int, topo: int = DUAL) -> dict:
     arrs = {k: np.zeros(p, dtype=np.int32)
             for k in ("parent", "child0", "child1", "dual", "depth")}
     ip = ctypes.POINTER(ctypes.c_int)
-    _check(lib().orc_trees(p, *[arrs[k].ctypes.data_as(ip) for k in
-                                ("parent", "child0", "child1", "dual",
-                                 "depth")]))
+    _check(lib().orc_trees_topo(p, topo, *[arrs[k].ctypes.data_as(ip) for k in
+                                           ("parent", "child0", "child1", "dual",
+                                            "depth")]))
     return arrs
 
 
@@ -123,8 +134,11 @@ def left_fold(x: np.ndarray, dt: int) -> np.ndarray:
     return _fold(lib().orc_left_fold, x, dt)
 
 
-def tree_fold(x: np.ndarray, dt: int) -> np.ndarray:
-    return _fold(lib().orc_tree_fold, x, dt)
+def tree_fold(x: np.ndarray, dt: int, topo: int = DUAL) -> np.ndarray:
+    x, p, m = _shape(x, dt)
+    y = np.empty(x.shape[1:], dtype=x.dtype)
+    _check(lib().orc_tree_fold_topo(p, topo, m, dt, _ptr(x), _ptr(y)))
+    return y
 
 
 def allreduce(x: np.ndarray, dt: int, out: np.ndarray | None = None):
@@ -134,14 +148,14 @@ def allreduce(x: np.ndarray, dt: int, out: np.ndarray | None = None):
     return y
 
 
-def simulate(x: np.ndarray, dt: int, b: int):
+def simulate(x: np.ndarray, dt: int, b: int, topo: int = DUAL):
     """Run the event-level simulation; returns (Y [p][m...], stats, last_round)."""
     x, p, m = _shape(x, dt)
     y = np.empty_like(x)
     stats = (ctypes.c_int64 * 6)()
     last = np.zeros(p, dtype=np.int32)
-    _check(lib().orc_simulate(p, m, b, dt, _ptr(x), _ptr(y), stats,
-                              last.ctypes.data_as(ctypes.POINTER(ctypes.c_int))))
+    _check(lib().orc_simulate_topo(p, topo, m, b, dt, _ptr(x), _ptr(y), stats,
+                                   last.ctypes.data_as(ctypes.POINTER(ctypes.c_int))))
     st = dict(zip(("steps", "first_block_last", "exchanges",
                    "max_ops_nonroot", "max_ops_root", "void_skipped"),
                   [int(v) for v in stats]))

@@ -122,23 +122,28 @@ def test_tree_equals_left_for_exact_ops(orc, p):
     assert (orc.tree_fold(xm, orc.MAT) == orc.left_fold(xm, orc.MAT)).all()
 
 
-def _golden_fp32():
+def _golden_fp32(which="dual"):
     for line in open(os.path.join(GOLD, "fp32_bracketing.txt")):
         if not line.strip() or line.startswith("#"):
             continue
         p, xs, y, why = [f.strip() for f in line.split(";")]
+        topo = "single" if p.startswith("single") else "dual"
+        if topo != which:
+            continue
+        p = int(p.split()[-1])
         x = np.array([float.fromhex(v) if v != "0" else 0.0 for v in xs.split()],
-                     dtype=np.float32).reshape(int(p), 1)
-        yield int(p), x, np.float32(float.fromhex(y)), why
+                     dtype=np.float32).reshape(p, 1)
+        yield p, x, np.float32(float.fromhex(y)), why
 
 
 def test_fp32_golden_bracketing(orc):
     n = 0
-    for p, x, y, why in _golden_fp32():
-        got = orc.tree_fold(x, orc.F32)[0]
-        assert got.tobytes() == y.tobytes(), (p, why, float(got).hex())
-        n += 1
-    assert n >= 7
+    for which, topo in (("dual", orc.DUAL), ("single", orc.SINGLE)):
+        for p, x, y, why in _golden_fp32(which):
+            got = orc.tree_fold(x, orc.F32, topo)[0]
+            assert got.tobytes() == y.tobytes(), (which, p, why, float(got).hex())
+            n += 1
+    assert n >= 9
 
 
 def test_fp32_golden_differs_from_left_fold(orc):
