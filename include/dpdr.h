@@ -14,9 +14,10 @@
  * two post-order-numbered complete binary trees, tree 0 = ranks
  * [0, floor(p/2)) and tree 1 = [floor(p/2), p); the value of node i is
  * v(child_1) (.) ( v(child_0) (.) x_i ) with child_0 = i-1, and
- * y = v(r0) (.) v(r1) for the roots r0 = floor(p/2)-1 and r1 = p-1.  Every
- * entry point below produces exactly this result, bit for bit, for every
- * element type (float32 included), in every y[i].
+ * y = v(r0) (.) v(r1) for the roots r0 = floor(p/2)-1 and r1 = p-1 (or, for
+ * a plan made with DPDR_TOPO_SINGLE, y = v(p-1) of one tree).  Every entry
+ * point below produces exactly this result, bit for bit, for every element
+ * type (float32 included), in every y[i].
  *
  * Conventions for all functions:
  *   - Status codes (dpdr_status) are returned; nothing throws, the device
@@ -66,6 +67,17 @@ typedef enum {
     DPDR_ERR_OOM = 5               /* device or pinned host memory exhausted */
 } dpdr_status;
 
+/* How the ranks are arranged.  DPDR_TOPO_DUAL is the paper's method: two
+ * post-order trees whose roots are duals (Sec. 1.1, Algorithm 1).
+ * DPDR_TOPO_SINGLE is the one-tree variant Sec. 1.2 discusses: all p ranks
+ * in one complete post-order tree, root p-1, no dual-root step (every
+ * non-leaf applies (.) at most twice per round); y = v(p-1), a different
+ * float32 bracketing from the dual trees'. */
+typedef enum {
+    DPDR_TOPO_DUAL = 0,
+    DPDR_TOPO_SINGLE = 1
+} dpdr_topology;
+
 /* Opaque plan; owns the device-side tables and scratch of one (p, m, type). */
 typedef struct dpdr_plan_s* dpdr_plan_t;
 
@@ -84,6 +96,10 @@ typedef struct CUstream_st* dpdr_stream_t;
  * rounds j = 0..b+d_i).  Any pointer may be NULL.  p >= 1. */
 int dpdr_tree(int p, int* parent, int* child0, int* child1, int* dual,
               int* depth);
+
+/* dpdr_tree for either topology (with DPDR_TOPO_SINGLE every dual is -1). */
+int dpdr_tree_topo(int p, dpdr_topology topo, int* parent, int* child0,
+                   int* child1, int* dual, int* depth);
 
 /* Block partition of Algorithm 1 (Sec. 1.1: b successive blocks of roughly
  * m/b elements): writes b+1 caller-owned starts, block j = [starts[j],
@@ -107,6 +123,12 @@ int dpdr_block_count_rule(int p, int64_t m, double kappa);
  * b is clamped to [1, max(m,1)].  p >= 1, m >= 0.  Returns NULL on error
  * (see dpdr_last_error).  Not thread-safe with respect to one plan. */
 dpdr_plan_t dpdr_plan(int p, int64_t m, dpdr_dtype dtype, dpdr_op op, int b);
+
+/* dpdr_plan for either topology (dpdr_plan is DPDR_TOPO_DUAL).  Every entry
+ * point then computes that topology's bracketing.  The allocation-free entry
+ * point supports the dual topology only. */
+dpdr_plan_t dpdr_plan_topo(int p, int64_t m, dpdr_dtype dtype, dpdr_op op,
+                           int b, dpdr_topology topo);
 
 /* Copies the plan's trees (caller-owned int[p] arrays, any may be NULL) and
  * the block count in use. */
@@ -159,7 +181,8 @@ int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
  *   [9] split layout cut depth  [10] its scratch rows (subtrees plus nodes
  *   above the cut)  [11] ranks per store
  *   group of its second kernel (0 when the split layout is not prepared)
- *   [12] CTAs per rank (column slices) of the schedule kernel */
+ *   [12] CTAs per rank (column slices) of the schedule kernel
+ *   [13] topology (dpdr_topology) */
 int dpdr_plan_info(dpdr_plan_t plan, int64_t* info, int n);
 
 /* Releases the plan's device and host memory.  The caller must first make

@@ -28,11 +28,14 @@ _IP = ctypes.POINTER(ctypes.c_int)
 _I64P = ctypes.POINTER(ctypes.c_int64)
 SIGNATURES = {
     "dpdr_tree": (ctypes.c_int, [ctypes.c_int, _IP, _IP, _IP, _IP, _IP]),
+    "dpdr_tree_topo": (ctypes.c_int, [ctypes.c_int, ctypes.c_int, _IP, _IP, _IP, _IP, _IP]),
     "dpdr_blocks": (ctypes.c_int, [ctypes.c_int64, ctypes.c_int, _I64P]),
     "dpdr_block_count_rule": (ctypes.c_int, [ctypes.c_int, ctypes.c_int64,
                                              ctypes.c_double]),
     "dpdr_plan": (_P, [ctypes.c_int, ctypes.c_int64, ctypes.c_int,
                        ctypes.c_int, ctypes.c_int]),
+    "dpdr_plan_topo": (_P, [ctypes.c_int, ctypes.c_int64, ctypes.c_int,
+                            ctypes.c_int, ctypes.c_int, ctypes.c_int]),
     "dpdr_plan_query": (ctypes.c_int, [_P, _IP, _IP, _IP, _IP, _IP, _IP]),
     "dpdr_plan_set": (ctypes.c_int, [_P, ctypes.c_int, ctypes.c_int64]),
     "dpdr_plan_info": (ctypes.c_int, [_P, _I64P, ctypes.c_int]),
@@ -82,13 +85,17 @@ def _check(rc: int, where: str) -> None:
         raise DpdrError(rc, where)
 
 
-def tree(p: int) -> dict:
-    """Dual post-order trees (host only): parent, child0, child1, dual, depth."""
+TOPOLOGIES = {"dual": 0, "single": 1}
+
+
+def tree(p: int, topology="dual") -> dict:
+    """Post-order trees (host only): parent, child0, child1, dual, depth."""
+    t = TOPOLOGIES[topology] if isinstance(topology, str) else int(topology)
     out = {k: np.zeros(p, np.int32) for k in ("parent", "child0", "child1",
                                                "dual", "depth")}
-    _check(lib().dpdr_tree(p, *[out[k].ctypes.data_as(_IP) for k in
-                                ("parent", "child0", "child1", "dual",
-                                 "depth")]), "dpdr_tree")
+    _check(lib().dpdr_tree_topo(p, t, *[out[k].ctypes.data_as(_IP) for k in
+                                         ("parent", "child0", "child1", "dual",
+                                          "depth")]), "dpdr_tree")
     return out
 
 
@@ -134,11 +141,12 @@ DTYPES = {"int32": DPDR_INT32, "float32": DPDR_FLOAT32,
 class Plan:
     """A plan for p virtual ranks of m elements (``dpdr_plan``)."""
 
-    def __init__(self, p: int, m: int, dtype, b: int = 0):
+    def __init__(self, p: int, m: int, dtype, b: int = 0, topology="dual"):
         dt = DTYPES[dtype] if isinstance(dtype, str) else int(dtype)
         op = DPDR_OP_MATMUL if dt == DPDR_MAT2X2_U32 else DPDR_OP_SUM
+        topo = TOPOLOGIES[topology] if isinstance(topology, str) else int(topology)
         L = lib()
-        h = L.dpdr_plan(int(p), int(m), dt, op, int(b))
+        h = L.dpdr_plan_topo(int(p), int(m), dt, op, int(b), topo)
         if not h:
             raise DpdrError(L.dpdr_last_error(), "dpdr_plan")
         self._h = h
@@ -175,12 +183,13 @@ class Plan:
         return out
 
     def info(self) -> dict:
-        v = np.zeros(13, np.int64)
-        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), 13),
+        v = np.zeros(14, np.int64)
+        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), 14),
                "dpdr_plan_info")
         keys = ("p", "m", "b", "max_depth", "auto_mode", "sched_ctas",
                 "sched_ranks_per_cta", "scratch_bytes", "vector_path",
-                "split_depth", "split_subtrees", "split_group", "sched_slices")
+                "split_depth", "split_subtrees", "split_group", "sched_slices",
+                "topology")
         return {k: int(x) for k, x in zip(keys, v)}
 
     def set(self, key: int, value: int) -> None:

@@ -33,6 +33,7 @@ struct Plan {
     int64_t m = 0;
     int dtype = 0;
     int op = 0;
+    int topo = 0;              // DPDR_TOPO_DUAL or DPDR_TOPO_SINGLE
     int b = 1;
     size_t esize = 4;
     int device = 0;
@@ -41,7 +42,7 @@ struct Plan {
     // trees (Sec. 1.1)
     std::vector<int> parent, child0, child1, dual, depth;
     int max_depth = 0;
-    int r0 = -1, r1 = 0;
+    int r0 = -1, r1 = 0;       // roots (r0 = -1: one tree, no dual)
     std::vector<uint8_t> tape;                 // column-streaming fold
     std::vector<LevelNode> levels;             // tile fold
     std::vector<int> level_off;                // nlevels + 1
@@ -111,7 +112,7 @@ struct Plan {
 };
 
 // host-side builders (plan.cpp)
-void build_tree(int p, int* parent, int* child0, int* child1, int* dual,
+void build_tree(int p, int topo, int* parent, int* child0, int* child1, int* dual,
                 int* depth);
 int block_count_rule(int p, int64_t m, double kappa);
 

@@ -136,6 +136,7 @@ int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t m
     a.p = P->p;
     a.r0 = P->r0;
     a.r1 = P->r1;
+    a.dual = P->r0 >= 0 ? 1 : 0;
     const int epv = int(16 / P->esize);
     a.nvec = vec ? mc / epv : 0;
     a.scalar_base = a.nvec * epv;

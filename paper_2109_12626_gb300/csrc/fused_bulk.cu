@@ -172,7 +172,7 @@ fused_bulk_kernel(FusedArgs a)
             fold_step<U>(__ldg(a.tape + i), v, acc, slot, kBulkConsumers);
         }
         if (!ok) break;
-        const uint4 y = (p >= 2) ? U::op(slot[0], acc) : acc;
+        const uint4 y = a.dual ? U::op(slot[0], acc) : acc;
         // the stores that last read this result buffer (two tiles ago) must
         // have finished reading it
         if (tid == 0) bulk_wait_read1();

@@ -40,6 +40,7 @@ struct FusedArgs {
     int nlevels;
     int p;
     int r0, r1;
+    int dual;               // 1: y = v(r0) (.) v(r1); 0: one tree, y = v(p-1)
     int64_t nvec;           // 16-byte units
     int64_t nscalar;        // single elements after the vector units
     int64_t scalar_base;    // element index of the first single element
@@ -154,7 +155,7 @@ __device__ __forceinline__ void stream_column(const FusedArgs& a, int64_t u,
 #pragma unroll
         for (int k = 0; k < kStreamAhead; k++) cur[k] = nxt[k];
     }
-    const T y = (p >= 2) ? U::op(slot[0], acc) : acc;  // v(r0) (.) v(r1)
+    const T y = a.dual ? U::op(slot[0], acc) : acc;  // v(r0) (.) v(r1), or v(root)
 #pragma unroll 4
     for (int i = 0; i < p; i++) U::st(rank_ptr_w(a.y, i), u, y);
 }

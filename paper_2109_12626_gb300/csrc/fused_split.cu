@@ -76,7 +76,7 @@ __device__ __forceinline__ void split_finish_column(const FusedArgs& a, int r, i
 #pragma unroll
         for (int k = 0; k < kStreamAhead; k++) cur[k] = nxt[k];
     }
-    const T y = (a.p >= 2) ? U::op(slot[0], acc) : acc;
+    const T y = a.dual ? U::op(slot[0], acc) : acc;
     const int i1 = min(a.p, (r + 1) * a.group);
 #pragma unroll 4
     for (int i = r * a.group; i < i1; i++) U::st(rank_ptr_w(a.y, i), u, y);

@@ -69,7 +69,7 @@ __device__ __forceinline__ void tile_body(const FusedArgs& a, int64_t u0,
     }
     for (int c = tid; c < wu; c += bd) {
         const T v1 = tile[(a.r1 << lg_wu) + c];
-        tile[(p << lg_wu) + c] = (p >= 2) ? U::op(tile[(a.r0 << lg_wu) + c], v1) : v1;
+        tile[(p << lg_wu) + c] = a.dual ? U::op(tile[(a.r0 << lg_wu) + c], v1) : v1;
     }
     __syncthreads();
     for (int idx = tid; idx < n; idx += bd) {

@@ -84,10 +84,10 @@ static void subtree(int lo, int n, int up, int d, int* parent, int* c0,
     }
 }
 
-void build_tree(int p, int* parent, int* child0, int* child1, int* dual,
+void build_tree(int p, int topo, int* parent, int* child0, int* child1, int* dual,
                 int* depth)
 {
-    const int n0 = p / 2;
+    const int n0 = topo == DPDR_TOPO_SINGLE ? 0 : p / 2;
     subtree(0, n0, -1, 0, parent, child0, child1, depth);
     subtree(n0, p - n0, -1, 0, parent, child0, child1, depth);
     for (int i = 0; i < p; i++) dual[i] = -1;
@@ -118,17 +118,25 @@ int block_count_rule(int p, int64_t m, double kappa)
 using namespace dpdr;
 
 // ------------------------------------------------------------- host ABI
-extern "C" int dpdr_tree(int p, int* parent, int* child0, int* child1,
-                         int* dual, int* depth)
+extern "C" int dpdr_tree_topo(int p, dpdr_topology topo, int* parent, int* child0,
+                              int* child1, int* dual, int* depth)
 {
     if (p < 1) return fail(DPDR_ERR_INVALID, "dpdr_tree: p < 1");
+    if (topo != DPDR_TOPO_DUAL && topo != DPDR_TOPO_SINGLE)
+        return fail(DPDR_ERR_INVALID, "dpdr_tree: unknown topology");
     std::vector<int> t(size_t(5) * size_t(p));
     int* T = t.data();
-    build_tree(p, T, T + p, T + 2 * p, T + 3 * p, T + 4 * p);
+    build_tree(p, topo, T, T + p, T + 2 * p, T + 3 * p, T + 4 * p);
     int* outs[5] = {parent, child0, child1, dual, depth};
     for (int k = 0; k < 5; k++)
         if (outs[k]) std::memcpy(outs[k], T + size_t(k) * p, sizeof(int) * p);
     return DPDR_OK;
+}
+
+extern "C" int dpdr_tree(int p, int* parent, int* child0, int* child1,
+                         int* dual, int* depth)
+{
+    return dpdr_tree_topo(p, DPDR_TOPO_DUAL, parent, child0, child1, dual, depth);
 }
 
 extern "C" int dpdr_blocks(int64_t m, int b, int64_t* starts)
@@ -180,10 +188,10 @@ static void build_tables(Plan* P)
     P->child1.assign(p, -1);
     P->dual.assign(p, -1);
     P->depth.assign(p, 0);
-    build_tree(p, P->parent.data(), P->child0.data(), P->child1.data(),
+    build_tree(p, P->topo, P->parent.data(), P->child0.data(), P->child1.data(),
                P->dual.data(), P->depth.data());
     P->max_depth = *std::max_element(P->depth.begin(), P->depth.end());
-    P->r0 = p / 2 - 1;
+    P->r0 = P->topo == DPDR_TOPO_SINGLE ? -1 : p / 2 - 1;
     P->r1 = p - 1;
 
     // tape of the column-streaming fold
@@ -288,6 +296,16 @@ static int allocate(Plan* P)
 extern "C" dpdr_plan_t dpdr_plan(int p, int64_t m, dpdr_dtype dtype,
                                  dpdr_op op, int b)
 {
+    return dpdr_plan_topo(p, m, dtype, op, b, DPDR_TOPO_DUAL);
+}
+
+extern "C" dpdr_plan_t dpdr_plan_topo(int p, int64_t m, dpdr_dtype dtype, dpdr_op op,
+                                      int b, dpdr_topology topo)
+{
+    if (topo != DPDR_TOPO_DUAL && topo != DPDR_TOPO_SINGLE) {
+        fail(DPDR_ERR_INVALID, "dpdr_plan: unknown topology");
+        return nullptr;
+    }
     if (p < 1 || m < 0) {
         fail(DPDR_ERR_INVALID, "dpdr_plan: need p >= 1 and m >= 0");
         return nullptr;
@@ -309,6 +327,7 @@ extern "C" dpdr_plan_t dpdr_plan(int p, int64_t m, dpdr_dtype dtype,
     }
     P->p = p;
     P->m = m;
+    P->topo = topo;
     P->dtype = dtype;
     P->op = op;
     P->esize = dtype == DPDR_MAT2X2_U32 ? 16 : 4;
@@ -421,7 +440,7 @@ extern "C" int dpdr_plan_info(dpdr_plan_t h, int64_t* info, int n)
                          P->sched_ctas, P->sched_ranks_per_cta,
                          int64_t(P->dmem_bytes + P->d_split_bytes), P->last_vector_path,
                          P->split_s, P->split_nseg, P->split_group,
-                         P->sched_slices_used};
+                         P->sched_slices_used, P->topo};
     const int k = int(sizeof v / sizeof v[0]);
     for (int i = 0; i < n; i++) info[i] = i < k ? v[i] : 0;
     return DPDR_OK;

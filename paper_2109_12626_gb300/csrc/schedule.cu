@@ -33,7 +33,8 @@
 // their ranks in increasing order inside each round.  Every wait is then on
 // a lower rank of the same round, on an earlier round, or (r0 only) on the
 // dual r1 whose partial depends on tree 1 alone, so with all CTAs resident
-// (cooperative launch) the schedule cannot deadlock.  Each wait is bounded
+// (cooperative launch) the schedule cannot deadlock.  With one tree (no
+// dual) the root's partial block j is final and is published down at once.  Each wait is bounded
 // in time; an expired wait records {rank, round, step} in the plan's error
 // word, raises an abort flag that ends every other wait, and returns.
 #include <algorithm>
@@ -229,7 +230,7 @@ __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j, int 
     const char* xi = reinterpret_cast<const char*>(__ldg(reinterpret_cast<const unsigned long long*>(a.x) + i));
     char* yi = reinterpret_cast<char*>(__ldg(reinterpret_cast<const unsigned long long*>(a.y) + i));
     const bool root = par < 0;
-    const bool paired_root = root && a.p >= 2;
+    const bool paired_root = root && a.r0 >= 0;
     const bool inb = j < a.b;
     const int64_t bs = inb ? blk_start(a, j) : 0, be = inb ? blk_start(a, j + 1) : 0;
     const int64_t s = slice_at<EPV>(a, bs, be, g), e = slice_at<EPV>(a, bs, be, g + 1);
@@ -269,11 +270,13 @@ __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j, int 
         publish(a, down + i, uint32_t(j + 1), i);
         return true;
     }
-    if (root) {  // p == 1: one processor, y = x
-        if (inb && xi != yi) {
+    if (root) {  // the root of a single tree (or p == 1): its block is final
+        if (!inb) return true;
+        if (!have && xi != yi) {
             block_op<Op>(a, yi, nullptr, xi, s, e);
             __syncthreads();
         }
+        publish(a, down + i, uint32_t(j + 1), i);
         return true;
     }
     // step 3 elsewhere: partial Y[j] up (in y_i, or x_i for a leaf), final
@@ -335,7 +338,8 @@ int schedule_configure(Plan* P)
         &occ, kernel_for(P->dtype), P->sched_threads, 0);
     if (e != cudaSuccess) return cuda_fail(e, "schedule occupancy");
     const int64_t kmax = int64_t(occ) * P->num_sms;
-    const int n0 = P->p / 2, n1 = P->p - n0;
+    // rank chunks never straddle the two trees (one tree: n0 = 0)
+    const int n0 = P->r0 >= 0 ? P->p / 2 : 0, n1 = P->p - n0;
     auto ctas = [&](int r) { return (n0 + r - 1) / r + (n1 + r - 1) / r; };
     // with a fixed number of slices, ranks per CTA must make room for them
     const int64_t per_chunk = std::max(1, P->sched_slices);

@@ -99,3 +99,11 @@ def test_status_strings(native):
     for s in range(6):
         assert L.dpdr_status_string(s)
     assert b"unknown" in L.dpdr_status_string(99)
+
+
+@pytest.mark.parametrize("p", list(range(1, 80)) + [1023, 1152, 4097])
+def test_single_tree_matches_oracle(native, orc, p):
+    a = native.tree(p, "single")
+    o = orc.trees(p, orc.SINGLE)
+    for k in ("parent", "child0", "child1", "dual", "depth"):
+        assert np.array_equal(a[k], o[k]), k
