@@ -294,21 +294,24 @@ def run_reference(args, w) -> dict:
 
 
 # -------------------------------------------------------------- sweeps
-def model_rounds(p: int) -> int:
+def model_rounds(p: int, topology: str = "dual") -> int:
     """Unit steps before the first block reaches the last leaf in the
-    schedule's rendezvous model (4h-7 for p = 2^h - 2, h >= 3)."""
+    schedule's rendezvous model: 4h-7 for dual trees with p = 2^h - 2
+    (h >= 3), 4h-4 for one tree with p = 2^h - 1 (the oracle's simulation
+    gives both)."""
+    extra = 1 if topology == "single" else 2
     h = 0
-    while (1 << h) < p + 2:
+    while (1 << h) < p + extra:
         h += 1
-    return max(1, 4 * h - 7)
+    return max(1, 4 * h - (4 if topology == "single" else 7))
 
 
-def fit_cost_model(p: int, m: int, points):
+def fit_cost_model(p: int, m: int, points, topology: str = "dual"):
     """Least-squares fit of T(b) = T0 + (L + 3(b-1)) (alpha + beta m / b)
     (Sec. 1.2's cost model plus a launch constant T0) to (b, seconds)
     points; returns T0, alpha, beta (seconds, seconds/element)."""
     import numpy as np
-    L = model_rounds(p)
+    L = model_rounds(p, topology)
     A = np.array([[1.0, L + 3 * (b - 1), (L + 3 * (b - 1)) * m / b] for b, _ in points])
     y = np.array([t for _, t in points])
     try:  # the constants are times: fit them non-negative
@@ -365,8 +368,9 @@ def run_sweep(args, w) -> int:
             ww = dict(w, m=m)
             xs = gen_device_inputs(ww, dev)
             ys = [torch.empty_like(x) for x in xs]
-            rec = {"sweep": "m", "workload": args.workload, "p": p, "m": m}
-            with pkg.Plan(p, m, kind, 0) as plan:
+            rec = {"sweep": "m", "workload": args.workload, "p": p, "m": m,
+                   "topology": args.topology}
+            with pkg.Plan(p, m, kind, 0, topology=args.topology) as plan:
                 bd = plan.bind(xs, ys)
                 t = _timed(lambda: bd.allreduce(), 20, None, graph=True)
                 info = plan.info()
@@ -389,20 +393,22 @@ def run_sweep(args, w) -> int:
     bs = sorted(set(int(v) for v in args.blist.split(",") if int(v) <= max(m, 1)))
     points = []
     for b in bs:
-        with pkg.Plan(p, m, kind, b) as plan:
+        with pkg.Plan(p, m, kind, b, topology=args.topology) as plan:
             bd = plan.bind(xs, ys)
             t = _timed(lambda: bd.allreduce_schedule(), 5 if m >= (1 << 20) else 10, None)
             plan.sync()
             points.append((b, t))
-            print(json.dumps({"sweep": "b", "workload": args.workload, "p": p, "m": m, "b": b,
+            print(json.dumps({"sweep": "b", "workload": args.workload, "topology": args.topology,
+                              "p": p, "m": m, "b": b,
                               "us": round(t * 1e6, 2), "slices": plan.info()["sched_slices"]}),
                   flush=True)
-    t0, alpha, beta = fit_cost_model(p, m, points)
+    t0, alpha, beta = fit_cost_model(p, m, points, args.topology)
     best = min(points, key=lambda x: x[1])
     kappa = alpha / beta if beta > 0 else float("inf")
     rule = pkg.block_count_rule(p, m, kappa) if beta > 0 and alpha > 0 else None
-    print(json.dumps({"sweep": "b-fit", "workload": args.workload, "p": p, "m": m,
-                      "rounds_L": model_rounds(p), "T0_us": round(t0 * 1e6, 3),
+    print(json.dumps({"sweep": "b-fit", "workload": args.workload, "topology": args.topology,
+                      "p": p, "m": m,
+                      "rounds_L": model_rounds(p, args.topology), "T0_us": round(t0 * 1e6, 3),
                       "alpha_us": round(alpha * 1e6, 4), "beta_ns_per_elem": round(beta * 1e9, 5),
                       "kappa_elems": round(kappa, 1) if beta > 0 else None,
                       "best_b": best[0], "best_us": round(best[1] * 1e6, 2),
@@ -430,11 +436,16 @@ def main(argv=None) -> int:
     ap.add_argument("--sweep", choices=("m", "b"), default=None,
                     help="m: all m = 2^k up to --m; b: schedule time against b")
     ap.add_argument("--blist", default="1,2,4,8,16,32,64,128,256,512,1024")
+    ap.add_argument("--topology", choices=("dual", "single"), default="dual",
+                    help="dual roots (the paper's method) or one tree (Sec. 1.2 variant)")
+    ap.add_argument("--p", type=int, default=None, help="override p (sweeps)")
     args = ap.parse_args(argv)
     args.warmup = max(args.warmup, 3)
 
     world, rank, local = dist_env()
     w = workload(args.workload, args.m)
+    if args.p:
+        w["p"] = int(args.p)
 
     if args.impl == "reference":
         if rank == 0:
@@ -461,7 +472,7 @@ def main(argv=None) -> int:
     b = args.b if args.b is not None else (w.get("b") or 0)
     xs = gen_device_inputs(w, dev)
     ys = [torch.empty_like(x) for x in xs]
-    plan = pkg.Plan(p, m, kind, b)
+    plan = pkg.Plan(p, m, kind, b, topology=args.topology)
     if args.split_depth is not None:
         plan.set(pkg.OPT_SPLIT_DEPTH, args.split_depth)
     if args.mode:
@@ -557,6 +568,7 @@ def main(argv=None) -> int:
         "scaling": "weak", "vs_baseline": None, "dtype": DTYPE_TAG[kind],
         "data": "synthetic (seeded counter-based generator, generated on device)",
         "config": {"workload": args.workload, "p": p, "m": m, "kind": kind,
+                   "topology": args.topology,
                    "kernel": args.kernel, "b": info["b"],
                    "fused_mode": args.mode or info["auto_mode"],
                    "split_depth": info["split_depth"] if (args.mode or info["auto_mode"]) == 3 else None,

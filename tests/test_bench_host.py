@@ -99,6 +99,7 @@ def test_cost_model_fit_recovers_known_constants():
     T0, alpha, beta = 8e-6, 2.5e-6, 0.4e-9
     L = bench.model_rounds(p)
     assert L == 4 * 11 - 7
+    assert bench.model_rounds(1023, "single") == 4 * 10 - 4
     pts = [(b, T0 + (L + 3 * (b - 1)) * (alpha + beta * m / b)) for b in (1, 4, 16, 64, 256, 1024)]
     t0, a, bta = bench.fit_cost_model(p, m, pts)
     assert t0 == pytest.approx(T0, rel=1e-6) and a == pytest.approx(alpha, rel=1e-6)
