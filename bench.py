@@ -45,8 +45,8 @@ if ROOT not in sys.path:
 
 DEFAULT_WORKLOAD = "p32_m134217728_f32"
 METRIC = "allreduce GB/s (p*m*sizeof read + p*m*sizeof written)"
-ESIZE = {"int32": 4, "float32": 4, "mat2x2u32": 16}
-DTYPE_TAG = {"int32": "int32", "float32": "f32", "mat2x2u32": "u32"}
+ESIZE = {"int32": 4, "float32": 4, "mat2x2u32": 16, "mat2x2f32": 16}
+DTYPE_TAG = {"int32": "int32", "float32": "f32", "mat2x2u32": "u32", "mat2x2f32": "f32"}
 # source files whose change invalidates a layout's measured DRAM traffic
 KERNEL_SOURCES = {"stream": ("fused_stream.cu", "fused_common.cuh"),
                   "tile": ("fused_tile.cu", "fused_common.cuh"),
@@ -241,7 +241,7 @@ def cpu_sample(w: dict, target_s: float = 12.0, max_cols: int | None = None):
     kw = I.workload_kwargs(w)
     x = torch.stack([I.rank_values(kind, w["seed"], i, cols, **kw) for i in range(p)])
     x = x.numpy()
-    dt = {"int32": O.I32, "float32": O.F32, "mat2x2u32": O.MAT}[kind]
+    dt = {"int32": O.I32, "float32": O.F32, "mat2x2u32": O.MAT, "mat2x2f32": O.MATF}[kind]
     if kind == "mat2x2u32":
         x = x.view(np.uint32).reshape(p, cols, 4)
     y = np.empty_like(x)
@@ -269,7 +269,7 @@ def run_reference(args, w) -> dict:
     cols = max(1, min(w["m"], (1 << 22) // p))
     kw = I.workload_kwargs(w)
     x = torch.stack([I.rank_values(kind, w["seed"], i, cols, **kw) for i in range(p)]).numpy()
-    dt = {"int32": O.I32, "float32": O.F32, "mat2x2u32": O.MAT}[kind]
+    dt = {"int32": O.I32, "float32": O.F32, "mat2x2u32": O.MAT, "mat2x2f32": O.MATF}[kind]
     if kind == "mat2x2u32":
         x = x.view(np.uint32).reshape(p, cols, 4)
     y = np.empty_like(x)

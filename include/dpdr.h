@@ -47,13 +47,17 @@ extern "C" {
 typedef enum {
     DPDR_INT32 = 0,      /* int32, sum wraps mod 2^32                       */
     DPDR_FLOAT32 = 1,    /* IEEE float32, sum rounded to nearest even        */
-    DPDR_MAT2X2_U32 = 2  /* 2x2 uint32 matrix, row-major a,b,c,d (16 bytes) */
+    DPDR_MAT2X2_U32 = 2, /* 2x2 uint32 matrix, row-major a,b,c,d (16 bytes) */
+    DPDR_MAT2X2_F32 = 3  /* 2x2 float32 matrix, row-major (16 bytes); each
+                            product entry is two rounded products and one
+                            rounded sum, never fused                        */
 } dpdr_dtype;
 
 typedef enum {
     DPDR_OP_SUM = 0,     /* with DPDR_INT32 or DPDR_FLOAT32                  */
-    DPDR_OP_MATMUL = 1   /* with DPDR_MAT2X2_U32: product mod 2^32, the lower
-                            rank on the left (non-commutative)              */
+    DPDR_OP_MATMUL = 1   /* with DPDR_MAT2X2_U32 (product mod 2^32) or
+                            DPDR_MAT2X2_F32: the lower rank on the left
+                            (non-commutative)                               */
 } dpdr_op;
 
 typedef enum {

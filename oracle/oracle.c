@@ -20,7 +20,9 @@
  *
  * Element types: int32 sum (wrapping two's complement, computed as uint32),
  * float32 sum (IEEE round-to-nearest-even, no contraction), 2x2 uint32 matrix
- * product mod 2^32 (row-major a b / c d, lower rank on the left), and an
+ * product mod 2^32 (row-major a b / c d, lower rank on the left), 2x2
+ * float32 matrix product (each entry two rounded products and a rounded
+ * sum: non-commutative and, in rounding, non-associative), and an
  * oracle-only "interval witness" whose elements are rank intervals [lo,hi]:
  * [a,b] (.) [b+1,c] = [a,c], every other pair gives the absorbing value
  * bottom = (-1,-1).  The witness is associative and non-commutative and fails
@@ -42,7 +44,7 @@
 #include <stdlib.h>
 #include <string.h>
 
-enum { ORC_I32 = 0, ORC_F32 = 1, ORC_MAT = 2, ORC_WIT = 3 };
+enum { ORC_I32 = 0, ORC_F32 = 1, ORC_MAT = 2, ORC_WIT = 3, ORC_MATF = 4 };
 
 enum {
     ORC_OK = 0,
@@ -67,6 +69,7 @@ static size_t esize(int dt)
     case ORC_F32: return 4;
     case ORC_MAT: return 16;
     case ORC_WIT: return 8;
+    case ORC_MATF: return 16;
     default: return 0;
     }
 }
@@ -101,6 +104,22 @@ static void op1(int dt, const void* a, const void* b, void* out)
         C[1] = A[0] * B[1] + A[1] * B[3];
         C[2] = A[2] * B[0] + A[3] * B[2];
         C[3] = A[2] * B[1] + A[3] * B[3];
+        memcpy(out, C, 16);
+        break;
+    }
+    case ORC_MATF: {
+        /* [A0 A1; A2 A3] * [B0 B1; B2 B3] in float32: each entry is two
+         * rounded products and one rounded sum, nothing fused */
+        float A[4], B[4], C[4];
+        memcpy(A, a, 16);
+        memcpy(B, b, 16);
+        for (int r = 0; r < 2; r++)
+            for (int c = 0; c < 2; c++) {
+                volatile float u = A[2 * r] * B[c];
+                volatile float v = A[2 * r + 1] * B[2 + c];
+                volatile float w = u + v;
+                C[2 * r + c] = w;
+            }
         memcpy(out, C, 16);
         break;
     }

@@ -3,7 +3,8 @@
 TEST INFRASTRUCTURE ONLY: the tests, the smoke check and the benchmark's CPU
 baseline use it; the product package never imports it.  Arrays are numpy,
 row-major ``[p][m]`` (``[p][m][4]`` uint32 words for 2x2 matrices,
-``[p][m][2]`` int32 for the interval witness).
+``[p][m][2]`` int32 for the interval witness, ``[p][m][4]`` float32 for
+2x2 float32 matrices).
 
 Functions and the passages they follow:
   trees(p, topo)           dual post-order trees, Sec. 1.1 (topo SINGLE: the
@@ -22,9 +23,9 @@ import subprocess
 
 import numpy as np
 
-I32, F32, MAT, WIT = 0, 1, 2, 3
-_ESIZE = {I32: 4, F32: 4, MAT: 16, WIT: 8}
-_DTYPE = {I32: np.int32, F32: np.float32, MAT: np.uint32, WIT: np.int32}
+I32, F32, MAT, WIT, MATF = 0, 1, 2, 3, 4
+_ESIZE = {I32: 4, F32: 4, MAT: 16, WIT: 8, MATF: 16}
+_DTYPE = {I32: np.int32, F32: np.float32, MAT: np.uint32, WIT: np.int32, MATF: np.float32}
 
 ERRORS = {0: "ok", 1: "invalid", 2: "no memory", 3: "mismatch", 4: "deadlock"}
 
@@ -98,6 +99,8 @@ def _shape(x: np.ndarray, dt: int):
     x = np.ascontiguousarray(x)
     if dt == MAT:
         assert x.ndim == 3 and x.shape[2] == 4 and x.dtype == np.uint32
+    elif dt == MATF:
+        assert x.ndim == 3 and x.shape[2] == 4 and x.dtype == np.float32
     elif dt == WIT:
         assert x.ndim == 3 and x.shape[2] == 2 and x.dtype == np.int32
     else:

@@ -10,7 +10,8 @@ from __future__ import annotations
 
 from ._native import (DPDR_ERR_CUDA, DPDR_ERR_INVALID,  # noqa: F401
                       DPDR_ERR_NOT_COOPERATIVE, DPDR_ERR_OOM, DPDR_ERR_TIMEOUT,
-                      DPDR_FLOAT32, DPDR_INT32, DPDR_MAT2X2_U32, DPDR_OK,
+                      DPDR_FLOAT32, DPDR_INT32, DPDR_MAT2X2_F32,
+                      DPDR_MAT2X2_U32, DPDR_OK,
                       DPDR_OP_MATMUL, DPDR_OP_SUM, OPT_BLOCKS, OPT_FUSED_MODE,
                       OPT_HOST_CHUNK_BYTES,
                       OPT_SCHED_RANKS_PER_CTA, OPT_SCHED_SLICES,

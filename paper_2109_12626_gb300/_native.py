@@ -12,7 +12,7 @@ from typing import Sequence
 
 import numpy as np
 
-DPDR_INT32, DPDR_FLOAT32, DPDR_MAT2X2_U32 = 0, 1, 2
+DPDR_INT32, DPDR_FLOAT32, DPDR_MAT2X2_U32, DPDR_MAT2X2_F32 = 0, 1, 2, 3
 DPDR_OP_SUM, DPDR_OP_MATMUL = 0, 1
 (DPDR_OK, DPDR_ERR_INVALID, DPDR_ERR_CUDA, DPDR_ERR_TIMEOUT,
  DPDR_ERR_NOT_COOPERATIVE, DPDR_ERR_OOM) = range(6)
@@ -135,7 +135,7 @@ def _stream(stream) -> int:
 
 
 DTYPES = {"int32": DPDR_INT32, "float32": DPDR_FLOAT32,
-          "mat2x2u32": DPDR_MAT2X2_U32}
+          "mat2x2u32": DPDR_MAT2X2_U32, "mat2x2f32": DPDR_MAT2X2_F32}
 
 
 class Plan:
@@ -143,7 +143,7 @@ class Plan:
 
     def __init__(self, p: int, m: int, dtype, b: int = 0, topology="dual"):
         dt = DTYPES[dtype] if isinstance(dtype, str) else int(dtype)
-        op = DPDR_OP_MATMUL if dt == DPDR_MAT2X2_U32 else DPDR_OP_SUM
+        op = DPDR_OP_MATMUL if dt in (DPDR_MAT2X2_U32, DPDR_MAT2X2_F32) else DPDR_OP_SUM
         topo = TOPOLOGIES[topology] if isinstance(topology, str) else int(topology)
         L = lib()
         h = L.dpdr_plan_topo(int(p), int(m), dt, op, int(b), topo)

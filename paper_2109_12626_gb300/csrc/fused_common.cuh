@@ -174,6 +174,7 @@ int dispatch(Plan* P, FusedArgs a, cudaStream_t s)
     switch (P->dtype) {
     case DPDR_INT32: return L<SumI32>::run(P, a, s);
     case DPDR_FLOAT32: return L<SumF32>::run(P, a, s);
+    case DPDR_MAT2X2_F32: return L<MatF32>::run(P, a, s);
     default: return L<MatU32>::run(P, a, s);
     }
 }

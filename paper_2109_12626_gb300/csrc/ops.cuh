@@ -71,6 +71,33 @@ struct MatU32 {
     }
 };
 
+// 2x2 float32 matrices, row-major; every entry is two rounded products and
+// one rounded sum (never contracted into an FMA), so the result is defined
+// by the bracketing alone: non-commutative, and non-associative in rounding.
+struct MatF32 {
+    static constexpr int kEpv = 1;
+    static constexpr int kEsize = 16;
+    __device__ __forceinline__ static uint32_t dot(uint32_t a, uint32_t b, uint32_t c, uint32_t d)
+    {
+        const float u = __fmul_rn(__uint_as_float(a), __uint_as_float(b));
+        const float v = __fmul_rn(__uint_as_float(c), __uint_as_float(d));
+        return __float_as_uint(__fadd_rn(u, v));
+    }
+    __device__ __forceinline__ static uint4 vec(uint4 a, uint4 b)
+    {
+        return make_uint4(dot(a.x, b.x, a.y, b.z), dot(a.x, b.y, a.y, b.w),
+                          dot(a.z, b.x, a.w, b.z), dot(a.z, b.y, a.w, b.w));
+    }
+    __device__ __forceinline__ static void one(const uint32_t* a, const uint32_t* b, uint32_t* o)
+    {
+        const uint4 r = vec(make_uint4(a[0], a[1], a[2], a[3]), make_uint4(b[0], b[1], b[2], b[3]));
+        o[0] = r.x;
+        o[1] = r.y;
+        o[2] = r.z;
+        o[3] = r.w;
+    }
+};
+
 __device__ __forceinline__ int64_t lmin(int64_t a, int64_t b) { return a < b ? a : b; }
 
 // ------------------------------------------------------------ memory units

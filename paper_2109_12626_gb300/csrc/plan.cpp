@@ -311,7 +311,8 @@ extern "C" dpdr_plan_t dpdr_plan_topo(int p, int64_t m, dpdr_dtype dtype, dpdr_o
         return nullptr;
     }
     const bool sum_ok = (dtype == DPDR_INT32 || dtype == DPDR_FLOAT32) && op == DPDR_OP_SUM;
-    const bool mat_ok = dtype == DPDR_MAT2X2_U32 && op == DPDR_OP_MATMUL;
+    const bool mat_ok = (dtype == DPDR_MAT2X2_U32 || dtype == DPDR_MAT2X2_F32) &&
+                        op == DPDR_OP_MATMUL;
     if (!sum_ok && !mat_ok) {
         fail(DPDR_ERR_INVALID, "dpdr_plan: unsupported (dtype, op) pair");
         return nullptr;
@@ -330,7 +331,7 @@ extern "C" dpdr_plan_t dpdr_plan_topo(int p, int64_t m, dpdr_dtype dtype, dpdr_o
     P->topo = topo;
     P->dtype = dtype;
     P->op = op;
-    P->esize = dtype == DPDR_MAT2X2_U32 ? 16 : 4;
+    P->esize = (dtype == DPDR_MAT2X2_U32 || dtype == DPDR_MAT2X2_F32) ? 16 : 4;
     P->b = clamp_b(m, b == 0 ? block_count_rule(p, m, 0) : b);
     build_tables(P);
     if (P->max_depth > kMaxDepth) {

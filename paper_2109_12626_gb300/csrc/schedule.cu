@@ -320,6 +320,7 @@ const void* kernel_for(int dtype)
     switch (dtype) {
     case DPDR_INT32: return kernel_ptr<SumI32>();
     case DPDR_FLOAT32: return kernel_ptr<SumF32>();
+    case DPDR_MAT2X2_F32: return kernel_ptr<MatF32>();
     default: return kernel_ptr<MatU32>();
     }
 }
@@ -548,11 +549,12 @@ int schedule_noalloc(int p, int64_t m, int dtype, int op, int b, const void* con
     if (p > kNoAllocMaxRanks)
         return fail_c(DPDR_ERR_INVALID, "no-alloc: p exceeds DPDR_NOALLOC_MAX_RANKS");
     const bool sum_ok = (dtype == DPDR_INT32 || dtype == DPDR_FLOAT32) && op == DPDR_OP_SUM;
-    const bool mat_ok = dtype == DPDR_MAT2X2_U32 && op == DPDR_OP_MATMUL;
+    const bool mat_ok = (dtype == DPDR_MAT2X2_U32 || dtype == DPDR_MAT2X2_F32) &&
+                        op == DPDR_OP_MATMUL;
     if (!sum_ok && !mat_ok) return fail_c(DPDR_ERR_INVALID, "no-alloc: unsupported (dtype, op)");
     if (b < 0) return fail_c(DPDR_ERR_INVALID, "no-alloc: b < 0");
     if (!x || !y) return fail_c(DPDR_ERR_INVALID, "no-alloc: x or y is NULL");
-    const size_t esize = dtype == DPDR_MAT2X2_U32 ? 16 : 4;
+    const size_t esize = (dtype == DPDR_MAT2X2_U32 || dtype == DPDR_MAT2X2_F32) ? 16 : 4;
     int vec = 1;
     for (int i = 0; i < p; i++) {
         const uintptr_t a = reinterpret_cast<uintptr_t>(x[i]), c = reinterpret_cast<uintptr_t>(y[i]);

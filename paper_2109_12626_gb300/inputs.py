@@ -20,6 +20,8 @@ benchmark configurations ask for):
   uniform_int32(lo, hi)  Lemire's multiply-shift map of a 32-bit word onto
                          [lo, hi] (exact: product < 2^53)
   words_u32              raw uniform 32-bit words (2x2 uint32 matrices)
+  near_identity_f32      2x2 float32 matrices I + E, entries of E exact
+                         dyadics of magnitude <= 2^-7
   normal_f32(sigma)      Irwin-Hall sum of twelve uniform 16-bit integers,
                          centred and scaled to unit variance (the classic
                          "sum of 12 uniforms" normal approximation, tails
@@ -97,6 +99,19 @@ def words_u32(seed: int, rank: int, cols, k: int, device="cpu") -> torch.Tensor:
     return w.to(torch.int32)
 
 
+def near_identity_f32(seed: int, rank: int, cols, device="cpu") -> torch.Tensor:
+    """2x2 float32 matrices I + E, each entry of E an exact dyadic
+    k * 2^-22 with k uniform on [-2^15, 2^15) (|E| <= 2^-7), so products of
+    thousands of them stay in range; shape [len(cols), 4]."""
+    c = _cols(cols, device)
+    z = words64(seed, rank, c)
+    k = torch.stack([_shr(z, 16 * q) & 0xFFFF for q in range(4)], dim=1) - 32768
+    e = k.to(torch.float64) * 2.0**-22
+    e[:, 0] += 1.0
+    e[:, 3] += 1.0
+    return e.to(torch.float32)
+
+
 def normal_f32(seed: int, rank: int, cols, sigma: float = 1.0,
                device="cpu") -> torch.Tensor:
     """float32 values ~ N(0, sigma^2) (Irwin-Hall of 12 16-bit uniforms)."""
@@ -126,6 +141,8 @@ def rank_values(kind: str, seed: int, rank: int, cols, device="cpu",
         return normal_f32(seed, rank, cols, kw.get("sigma", 1.0), device)
     if kind == "mat2x2u32":
         return words_u32(seed, rank, cols, 4, device)
+    if kind == "mat2x2f32":
+        return near_identity_f32(seed, rank, cols, device)
     raise ValueError(kind)
 
 
@@ -145,6 +162,8 @@ WORKLOADS = {
     # p=32, m=134217728 float32 ~ N(0, 1e-3^2), sum
     "p32_m134217728_f32": dict(p=32, m=134217728, kind="float32", seed=5,
                                sigma=1e-3, b=1024),
+    # non-commutative float32: p=36, 2x2 float32 matrices near identity
+    "p36_m65536_mat2x2f32": dict(p=36, m=65536, kind="mat2x2f32", seed=6, b=16),
 }
 
 

@@ -7,8 +7,10 @@ import torch
 
 from paper_2109_12626_gb300 import inputs as I
 
-NP_DT = {"int32": np.int32, "float32": np.float32, "mat2x2u32": np.uint32}
-TORCH_DT = {"int32": torch.int32, "float32": torch.float32, "mat2x2u32": torch.int32}
+NP_DT = {"int32": np.int32, "float32": np.float32, "mat2x2u32": np.uint32,
+         "mat2x2f32": np.float32}
+TORCH_DT = {"int32": torch.int32, "float32": torch.float32, "mat2x2u32": torch.int32,
+            "mat2x2f32": torch.float32}
 
 
 def host_inputs(kind, seed, p, m, **kw):

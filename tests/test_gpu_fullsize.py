@@ -27,8 +27,10 @@ def pkg():
 
 
 def _device_inputs(w, m, dev):
+    """One tensor per rank: [m] for scalars, [m, 4] for 2x2 matrices (so a
+    column index picks a whole element)."""
     kw = I.workload_kwargs(w)
-    return [I.rank_values(w["kind"], w["seed"], i, m, device=dev, **kw).reshape(-1)
+    return [I.rank_values(w["kind"], w["seed"], i, m, device=dev, **kw).contiguous()
             for i in range(w["p"])]
 
 
@@ -50,10 +52,13 @@ def _sampled_check(orc, w, m, xs, ys, cols):
     kw = I.workload_kwargs(w)
     ct = torch.from_numpy(cols)
     host = torch.stack([I.rank_values(kind, w["seed"], i, ct, **kw) for i in range(p)])
-    dt = {"int32": orc.I32, "float32": orc.F32, "mat2x2u32": orc.MAT}[kind]
+    dt = {"int32": orc.I32, "float32": orc.F32, "mat2x2u32": orc.MAT,
+          "mat2x2f32": orc.MATF}[kind]
     hx = host.numpy()
     if kind == "mat2x2u32":
         hx = hx.view(np.uint32).reshape(p, len(cols), 4)
+    elif kind == "mat2x2f32":
+        hx = np.ascontiguousarray(hx).reshape(p, len(cols), 4)
     want = expect_bits(orc.tree_fold(hx, dt))
     cd = ct.to(xs[0].device)
     # the device generated the same inputs
@@ -70,6 +75,9 @@ def _sampled_check(orc, w, m, xs, ys, cols):
 @pytest.mark.parametrize("name,kernels", [
     ("p32_m134217728_f32", ("fused", "schedule")),
     ("p1152_m4194304_f32", ("fused", "schedule")),
+    ("p36_m65536_mat2x2u32", ("fused", "schedule")),
+    ("p36_m65536_mat2x2f32", ("fused", "schedule")),
+    ("p7_m1000_int32", ("fused", "schedule")),
 ])
 def test_full_size_workloads(pkg, orc, name, kernels):
     w = dict(I.WORKLOADS[name])

@@ -31,6 +31,9 @@ CASES = [
     ("p5_m1_int32", "int32", 6, 5, 1, dict(lo=-5, hi=5), [1]),
     ("p100_m77_mat", "mat2x2u32", 7, 100, 77, {}, [1, 7, 77]),
     ("p255_m2050_f32", "float32", 8, 255, 2050, {}, [3, 16]),
+    ("p36_m65536_matf", "mat2x2f32", 6, 36, 65536, {}, [16, 1, 7]),
+    ("p1152_m1025_matf", "mat2x2f32", 6, 1152, 1025, {}, [1, 4]),
+    ("p3_m9_matf", "mat2x2f32", 6, 3, 9, {}, [1, 9]),
 ]
 
 
@@ -43,7 +46,8 @@ def pkg():
 
 
 def _want(orc, x, kind):
-    dt = {"int32": orc.I32, "float32": orc.F32, "mat2x2u32": orc.MAT}[kind]
+    dt = {"int32": orc.I32, "float32": orc.F32, "mat2x2u32": orc.MAT,
+          "mat2x2f32": orc.MATF}[kind]
     return expect_bits(orc.tree_fold(x, dt))
 
 
@@ -108,7 +112,8 @@ def _run(pkg, plan, run, xs, ys):
 
 
 @pytest.mark.parametrize("kind,p,m", [("int32", 7, 1000), ("float32", 1152, 4099),
-                                      ("mat2x2u32", 36, 999), ("float32", 2, 5)])
+                                      ("mat2x2u32", 36, 999), ("float32", 2, 5),
+                                      ("mat2x2f32", 100, 513)])
 @pytest.mark.parametrize("run", RUNS)
 def test_in_place(pkg, orc, kind, p, m, run):
     """y[i] == x[i]: Algorithm 1 works in place (Y <- x_i, y ends in Y)."""
@@ -122,7 +127,8 @@ def test_in_place(pkg, orc, kind, p, m, run):
 
 
 @pytest.mark.parametrize("kind,p,m", [("int32", 7, 1001), ("float32", 1152, 133),
-                                      ("mat2x2u32", 36, 257), ("float32", 32, 9999)])
+                                      ("mat2x2u32", 36, 257), ("float32", 32, 9999),
+                                      ("mat2x2f32", 36, 257)])
 @pytest.mark.parametrize("run", RUNS)
 def test_four_byte_aligned_buffers(pkg, orc, kind, p, m, run):
     """Buffers only 4-byte aligned take the single-element paths."""

@@ -13,7 +13,7 @@ pytestmark = pytest.mark.gpu
 CASES = [("float32", 1, 33), ("float32", 2, 1001), ("int32", 3, 17), ("mat2x2u32", 5, 300),
          ("float32", 7, 4099), ("float32", 15, 65541), ("int32", 31, 2000),
          ("mat2x2u32", 63, 129), ("float32", 255, 3001), ("float32", 1023, 1027),
-         ("int32", 1152, 4099)]
+         ("int32", 1152, 4099), ("mat2x2f32", 127, 700)]
 
 
 @pytest.fixture(scope="module")
@@ -25,7 +25,8 @@ def pkg():
 
 
 def _want(orc, x, kind):
-    dt = {"int32": orc.I32, "float32": orc.F32, "mat2x2u32": orc.MAT}[kind]
+    dt = {"int32": orc.I32, "float32": orc.F32, "mat2x2u32": orc.MAT,
+          "mat2x2f32": orc.MATF}[kind]
     return expect_bits(orc.tree_fold(x, dt, orc.SINGLE))
 
 

@@ -179,3 +179,60 @@ def test_allreduce_copies_to_all_rows(orc):
     x = rng.integers(-1000, 1001, (7, 100), dtype=np.int64).astype(np.int32)
     y = orc.allreduce(x, orc.I32)
     assert (y == orc.tree_fold(x, orc.I32)[None, :]).all()
+
+
+def _read_fmats(line):
+    return [[float.fromhex(v) if v not in ("0", "-0") else 0.0 for v in t.split(",")]
+            for t in line.split()]
+
+
+def test_matf_golden(orc):
+    n = 0
+    for line in open(os.path.join(GOLD, "mat2x2_f32.txt")):
+        if not line.strip() or line.startswith("#"):
+            continue
+        p, xs, ys, why = [f.strip() for f in line.split(";")]
+        p = int(p)
+        x = np.array(_read_fmats(xs), dtype=np.float32).reshape(p, 1, 4)
+        want = np.array(_read_fmats(ys)[0], dtype=np.float32)
+        got = orc.tree_fold(x, orc.MATF)[0]
+        assert got.tobytes() == want.tobytes(), (why, got)
+        n += 1
+    assert n >= 2
+    # the p = 3 case is one where the bracketing decides the bits
+    x = np.array(_read_fmats("0x1.000002p+0,0,0,0x1p+0 0x1.fffffep-1,0,0,0x1p+0 "
+                             "0x1.fffffep-1,0,0,0x1p+0"), np.float32).reshape(3, 1, 4)
+    assert orc.left_fold(x, orc.MATF)[0, 0] == np.float32(1 - 2.0**-24)
+
+
+@pytest.mark.parametrize("p", [1, 2, 3, 7, 12])
+def test_matf_exact_on_small_integers(orc, p):
+    """Small non-negative integer matrices: every product and sum is exact in
+    float32, so the float32 product equals the uint32 product entry by entry
+    (this pins the entry formulas and the operand order)."""
+    rng = np.random.default_rng(100 + p)
+    xi = rng.integers(0, 2, (p, 6, 4), dtype=np.int64)
+    want = orc.left_fold(xi.astype(np.uint32), orc.MAT).astype(np.float64)
+    assert want.max() < 2**24
+    for f in (orc.left_fold, orc.tree_fold):
+        assert np.array_equal(f(xi.astype(np.float32), orc.MATF).astype(np.float64), want)
+
+
+@pytest.mark.parametrize("p", [2, 5, 16, 36])
+def test_matf_close_to_exact_product(orc, p):
+    """Near-identity float32 matrices: the tree-bracketed float32 product is
+    within a few ulp (relative 1e-5) of the exact product computed with
+    Python fractions."""
+    from fractions import Fraction
+    rng = np.random.default_rng(p)
+    x = (np.eye(2).reshape(1, 1, 4) + rng.integers(-2**15, 2**15, (p, 3, 4)) * 2.0**-22)
+    x = x.astype(np.float32)
+    y = orc.tree_fold(x, orc.MATF)
+    for e in range(3):
+        P = [[Fraction(1), Fraction(0)], [Fraction(0), Fraction(1)]]
+        for i in range(p):
+            Q = [[Fraction(float(x[i, e, 0])), Fraction(float(x[i, e, 1]))],
+                 [Fraction(float(x[i, e, 2])), Fraction(float(x[i, e, 3]))]]
+            P = [[P[r][0] * Q[0][c] + P[r][1] * Q[1][c] for c in range(2)] for r in range(2)]
+        ex = np.array([float(P[0][0]), float(P[0][1]), float(P[1][0]), float(P[1][1])])
+        assert np.allclose(y[e].astype(np.float64), ex, rtol=0, atol=1e-5 * p)
