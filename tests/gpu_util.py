@@ -55,7 +55,7 @@ def empty_like_ranks(xs, fill=-3, pad_front=0):
 
 def bits(t) -> np.ndarray:
     """Raw 32-bit words of a tensor (float32 compared bit for bit)."""
-    return t.detach().cpu().contiguous().view(torch.int32).numpy()
+    return t.detach().cpu().contiguous().view(torch.int32).numpy().reshape(-1)
 
 
 def expect_bits(want: np.ndarray) -> np.ndarray:
