@@ -137,29 +137,24 @@ __device__ __forceinline__ void stream_column(const FusedArgs& a, int64_t u,
 {
     using T = typename U::T;
     const int p = a.p;
-    T cur[kStreamAhead], nxt[kStreamAhead];
-#pragma unroll
-    for (int k = 0; k < kStreamAhead; k++)
-        if (k < p) cur[k] = U::ld(rank_ptr(a.x, k), u);
-    T acc = cur[0];
+    T acc{};  // set by rank 0, a leaf
+    // one batch of kStreamAhead loads in flight per thread; the other warps
+    // of the four CTAs per SM cover the latency between batches
     for (int i0 = 0; i0 < p; i0 += kStreamAhead) {
+        T cur[kStreamAhead];
 #pragma unroll
         for (int k = 0; k < kStreamAhead; k++)
-            if (i0 + kStreamAhead + k < p)
-                nxt[k] = U::ld(rank_ptr(a.x, i0 + kStreamAhead + k), u);
+            if (i0 + k < p) cur[k] = U::ld(rank_ptr(a.x, i0 + k), u);
         const unsigned long long tp =
             __ldg(reinterpret_cast<const unsigned long long*>(a.tape + i0));
 #pragma unroll
         for (int k = 0; k < kStreamAhead; k++)
             if (i0 + k < p) fold_step<U>(unsigned(tp >> (8 * k)) & 0xffu, cur[k], acc, slot, stride);
-#pragma unroll
-        for (int k = 0; k < kStreamAhead; k++) cur[k] = nxt[k];
     }
     const T y = a.dual ? U::op(slot[0], acc) : acc;  // v(r0) (.) v(r1), or v(root)
 #pragma unroll 4
     for (int i = 0; i < p; i++) U::st(rank_ptr_w(a.y, i), u, y);
 }
-
 
 // launchers, one per layout (dispatch on the plan's element type)
 int launch_stream(Plan* P, FusedArgs a, cudaStream_t s);

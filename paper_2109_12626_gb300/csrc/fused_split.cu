@@ -29,21 +29,15 @@ __device__ __forceinline__ void split_reduce_column(const FusedArgs& a, int g, i
         U::st_keep(row, u, U::ld(rank_ptr(a.x, lo), u));
         return;
     }
-    T cur[kStreamAhead], nxt[kStreamAhead];
-#pragma unroll
-    for (int k = 0; k < kStreamAhead; k++)
-        if (lo + k <= hi) cur[k] = U::ld(rank_ptr(a.x, lo + k), u);
-    T acc = cur[0];
+    T acc{};  // set by rank lo, a leaf
     for (int i0 = lo; i0 <= hi; i0 += kStreamAhead) {
+        T cur[kStreamAhead];
 #pragma unroll
         for (int k = 0; k < kStreamAhead; k++)
-            if (i0 + kStreamAhead + k <= hi)
-                nxt[k] = U::ld(rank_ptr(a.x, i0 + kStreamAhead + k), u);
+            if (i0 + k <= hi) cur[k] = U::ld(rank_ptr(a.x, i0 + k), u);
 #pragma unroll
         for (int k = 0; k < kStreamAhead; k++)
             if (i0 + k <= hi) fold_step<U>(__ldg(a.tape + i0 + k), cur[k], acc, slot, stride);
-#pragma unroll
-        for (int k = 0; k < kStreamAhead; k++) cur[k] = nxt[k];
     }
     U::st_keep(row, u, acc);
 }
@@ -54,27 +48,22 @@ __device__ __forceinline__ void split_finish_column(const FusedArgs& a, int r, i
 {
     using T = typename U::T;
     const int n = a.nitems;
-    T cur[kStreamAhead], nxt[kStreamAhead];
     // every item is a scratch row: a subtree value or a copied input, so
     // this kernel never reads an input that another CTA may be overwriting
     // with the result (in-place use)
     auto load = [&](int k) -> T {
         return U::ld_keep(a.part + int64_t(__ldg(&a.items[k].x)) * a.part_stride, u);
     };
-#pragma unroll
-    for (int k = 0; k < kStreamAhead; k++)
-        if (k < n) cur[k] = load(k);
-    T acc = cur[0];
+    T acc{};  // set by the first item, a subtree
     for (int k0 = 0; k0 < n; k0 += kStreamAhead) {
+        T cur[kStreamAhead];
 #pragma unroll
         for (int k = 0; k < kStreamAhead; k++)
-            if (k0 + kStreamAhead + k < n) nxt[k] = load(k0 + kStreamAhead + k);
+            if (k0 + k < n) cur[k] = load(k0 + k);
 #pragma unroll
         for (int k = 0; k < kStreamAhead; k++)
             if (k0 + k < n)
                 fold_step<U>(unsigned(__ldg(&a.items[k0 + k].y)) & 0xffu, cur[k], acc, slot, stride);
-#pragma unroll
-        for (int k = 0; k < kStreamAhead; k++) cur[k] = nxt[k];
     }
     const T y = a.dual ? U::op(slot[0], acc) : acc;
     const int i1 = min(a.p, (r + 1) * a.group);
@@ -83,7 +72,7 @@ __device__ __forceinline__ void split_finish_column(const FusedArgs& a, int r, i
 }
 
 template <class Op>
-__global__ void __launch_bounds__(kStreamThreads, 3)
+__global__ void __launch_bounds__(kStreamThreads, 4)
 fused_split_reduce_kernel(FusedArgs a)
 {
     extern __shared__ uint4 smem[];
@@ -98,7 +87,7 @@ fused_split_reduce_kernel(FusedArgs a)
 }
 
 template <class Op>
-__global__ void __launch_bounds__(kStreamThreads, 3)
+__global__ void __launch_bounds__(kStreamThreads, 4)
 fused_split_finish_kernel(FusedArgs a)
 {
     extern __shared__ uint4 smem[];

@@ -9,7 +9,7 @@ namespace fused {
 namespace {
 
 template <class Op>
-__global__ void __launch_bounds__(kStreamThreads, 3)
+__global__ void __launch_bounds__(kStreamThreads, 4)
 fused_stream_kernel(FusedArgs a)
 {
     extern __shared__ uint4 smem[];
