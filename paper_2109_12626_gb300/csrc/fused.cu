@@ -13,17 +13,17 @@ using fused::tile_lg_wu;
 static int64_t stream_target(const Plan* P) { return int64_t(P->num_sms) * 1024; }
 
 // Layout choice, from layout sweeps measured on GB300:
-//  * deep trees (p >= 128) with at least 8192 column units: the split layout,
+//  * deep trees (p >= 128) with at least 4096 column units: the split layout,
 //    whose read phase (first kernel) and write phase (second kernel) keep
-//    HBM traffic one-directional; it beats column streaming from m = 2^15 up
-//    to the largest sizes at p = 1152;
+//    HBM traffic one-directional; at p = 1152 it beats the tile from
+//    m = 2^14 and column streaming up to the largest sizes;
 //  * otherwise column streaming once there are a quarter of the columns it
 //    needs to fill the GPU (p = 36, 2x2 matrices, m = 2^16: 13 us against the
 //    tile's 15 us), and the shared-memory tile below that.
 int fused_auto_mode(const Plan* P)
 {
     const int64_t units = P->m * int64_t(P->esize) / 16;
-    if (P->p >= 128 && units >= 8192 && P->split_ready) return 3;
+    if (P->p >= 128 && units >= 4096 && P->split_ready) return 3;
     if (units >= stream_target(P) / 4) return 1;
     if (tile_lg_wu(P) >= 0) return 2;
     return P->split_ready ? 3 : 1;
@@ -34,7 +34,7 @@ int fused_auto_mode(const Plan* P)
 static bool split_wanted(const Plan* P)
 {
     const int64_t units = P->m * int64_t(P->esize) / 16;
-    return P->p >= 128 && units >= 8192;
+    return P->p >= 128 && units >= 4096;
 }
 
 // Split layout: cut depth s, subtree table, top-of-tree item list, rank
@@ -48,16 +48,18 @@ int fused_split_prepare(Plan* P, bool force, int depth)
     const int64_t units = std::max<int64_t>(1, P->m * int64_t(P->esize) / 16);
     const int64_t target = stream_target(P);
     // automatic cut: the shallowest depth whose subtrees give the first
-    // kernel four times the columns the GPU needs in flight, but no deeper
-    // than a third of the tree height (the second kernel's sequential walk
-    // over the nodes above the cut grows as 2^(s+1))
+    // kernel three times the columns the GPU needs in flight, but no deeper
+    // than 4 and than a third of the tree height plus one (the second
+    // kernel's sequential walk over the nodes above the cut grows as
+    // 2^(s+1)); measured best cuts at p = 1152: 4 at m = 2^14..2^15, 3 at
+    // 2^16, 2 at 2^17..2^18, 1 at 2^19..2^20, 0 above
     int s = depth;
     if (s < 0) {
-        const int cap = std::max(1, P->max_depth / 3);
+        const int cap = std::min(4, std::max(1, P->max_depth / 3 + 1));
         for (s = 0; s < cap; s++) {
             int64_t n = 0;
             for (int i = 0; i < p; i++) n += P->depth[i] == s;
-            if (n * units >= 4 * target) break;
+            if (n * units >= 3 * target) break;
         }
     }
     s = std::min(s, P->max_depth);
