@@ -47,21 +47,18 @@ int fused_split_prepare(Plan* P, bool force, int depth)
     if (p < 2) return DPDR_OK;  // one rank: nothing to split
     const int64_t units = std::max<int64_t>(1, P->m * int64_t(P->esize) / 16);
     const int64_t target = stream_target(P);
-    // automatic cut: the shallowest depth whose subtrees give the first
-    // kernel three times the columns the GPU needs in flight, but no deeper
-    // than 4 and than a third of the tree height plus one (the second
-    // kernel's sequential walk over the nodes above the cut grows as
-    // 2^(s+1)); measured best cuts at p = 1152: 4 at m = 2^14..2^15, 3 at
-    // 2^16, 2 at 2^17..2^18, 1 at 2^19..2^20, 0 above
+    // automatic cut, from the measured best cuts at p = 1152 (the first
+    // kernel wants many subtree columns, the second kernel's sequential walk
+    // over the 2^(s+2) - 2 rows grows with s): depth 4 below 16 K column
+    // units, 3 below 64 K, 2 below 256 K, 1 below 512 K, 0 above; never
+    // deeper than the tree allows
     int s = depth;
     if (s < 0) {
-        const int cap = std::min(4, std::max(1, P->max_depth / 3 + 1));
-        for (s = 0; s < cap; s++) {
-            int64_t n = 0;
-            for (int i = 0; i < p; i++) n += P->depth[i] == s;
-            if (n * units >= 3 * target) break;
-        }
+        s = units < (16 << 10) ? 4 : units < (64 << 10) ? 3 : units < (256 << 10) ? 2
+          : units < (512 << 10) ? 1 : 0;
+        s = std::min(s, std::max(0, P->max_depth - 2));
     }
+    (void)target;
     s = std::min(s, P->max_depth);
     if (P->split_ready && P->split_s == s) return DPDR_OK;
     if (!force && !split_wanted(P)) return DPDR_OK;
