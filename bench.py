@@ -439,6 +439,8 @@ def main(argv=None) -> int:
     ap.add_argument("--topology", choices=("dual", "single"), default="dual",
                     help="dual roots (the paper's method) or one tree (Sec. 1.2 variant)")
     ap.add_argument("--p", type=int, default=None, help="override p (sweeps)")
+    ap.add_argument("--host-path", type=int, default=0,
+                    help="e2e leg: 0 direct when possible, 1 copy pipeline, 2 direct")
     args = ap.parse_args(argv)
     args.warmup = max(args.warmup, 3)
 
@@ -533,6 +535,7 @@ def main(argv=None) -> int:
             h.copy_(x)
         for h in yh:
             h.zero_()
+        plan.set(pkg.OPT_HOST_PATH, args.host_path)
         for _ in range(2):
             plan.allreduce_host(xh, yh, xs, ys, stream)
         plan.sync(stream)
@@ -548,7 +551,9 @@ def main(argv=None) -> int:
         t2 = max_over_ranks(s2.elapsed_time(e2), world, dev) / k2
         e2e = {"value": round(world * algo_bytes / (t2 * 1e-3) / 1e9, 3), "unit": "GB/s",
                "h2d_bytes_per_step": p * m * es, "d2h_bytes_per_step": p * m * es,
-               "steps": k2, "ms_per_step": round(t2, 3), "host_numa_node": node}
+               "steps": k2, "ms_per_step": round(t2, 3), "host_numa_node": node,
+               "path": {1: "copy pipeline", 2: "direct (kernel on host memory)"}.get(
+                   plan.info()["host_path"], "?")}
         del xh, yh
         os.sched_setaffinity(0, saved)
 

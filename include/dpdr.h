@@ -163,8 +163,10 @@ int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
  *                             (0 = as many as fit co-resident, slices of at
  *                             least 1024 elements, at most 64)
  *   DPDR_OPT_HOST_CHUNK_BYTES bytes of rank data per column chunk of
- *                             dpdr_allreduce_host's pipeline (default 2^30,
- *                             minimum 4096) */
+ *                             dpdr_allreduce_host's copy pipeline (default
+ *                             2^30, minimum 4096)
+ *   DPDR_OPT_HOST_PATH        dpdr_allreduce_host: 0 direct when possible,
+ *                             else copy; 1 copy pipeline; 2 direct only */
 enum {
     DPDR_OPT_FUSED_MODE = 1,
     DPDR_OPT_WAIT_LIMIT_NS = 2,
@@ -174,7 +176,8 @@ enum {
     DPDR_OPT_BLOCKS = 6,
     DPDR_OPT_SPLIT_DEPTH = 7,
     DPDR_OPT_SCHED_SLICES = 8,
-    DPDR_OPT_HOST_CHUNK_BYTES = 9
+    DPDR_OPT_HOST_CHUNK_BYTES = 9,
+    DPDR_OPT_HOST_PATH = 10
 };
 int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
 
@@ -186,7 +189,8 @@ int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
  *   above the cut)  [11] ranks per store
  *   group of its second kernel (0 when the split layout is not prepared)
  *   [12] CTAs per rank (column slices) of the schedule kernel
- *   [13] topology (dpdr_topology) */
+ *   [13] topology (dpdr_topology)
+ *   [14] path of the last dpdr_allreduce_host: 1 copy pipeline, 2 direct */
 int dpdr_plan_info(dpdr_plan_t plan, int64_t* info, int n);
 
 /* Releases the plan's device and host memory.  The caller must first make
@@ -215,16 +219,23 @@ int dpdr_allreduce(dpdr_plan_t plan, const void* const* x, void* const* y,
 int dpdr_allreduce_schedule(dpdr_plan_t plan, const void* const* x,
                             void* const* y, dpdr_stream_t stream);
 
-/* Host buffers end to end: copies x_host[i] into the device buffers
- * x_dev[i], runs the fused kernel into y_dev, and copies y_dev[i] back into
- * y_host[i].  All four are host arrays of p pointers; the device buffers
- * follow dpdr_allreduce's rules.  The columns are cut into chunks (about
- * 1 GB of rank data each) that flow through a pipeline: copies in on one
- * plan-owned stream, the kernel on `stream`, copies out on another, so the
- * two copy directions and the kernel overlap (with pinned host memory;
- * pageable memory works but does not overlap).  The whole call is ordered
- * after earlier work on `stream`, and later work on `stream` waits for its
- * last copy. */
+/* Host buffers end to end: y_host[i] = x_host[0] (.) ... (.) x_host[p-1]
+ * for host memory x_host[i], y_host[i] (all four arguments are host arrays
+ * of p pointers).  Two paths:
+ *   direct  when the GPU can address every host buffer (pinned memory, or
+ *           pageable memory on systems whose GPU uses the CPU page tables,
+ *           such as Grace with NVLink-C2C): one launch of the column-
+ *           streaming fused kernel loads the inputs from host memory and
+ *           stores the result to host memory, both link directions at once;
+ *           x_dev and y_dev are not used and may be NULL.
+ *   copy    otherwise: the columns are cut into chunks (about 1 GB of rank
+ *           data each) that flow through a pipeline -- copies into the
+ *           device buffers x_dev[i] on one plan-owned stream, the kernel on
+ *           `stream` into y_dev, copies out on another stream -- so the two
+ *           copy directions and the kernel overlap.
+ * DPDR_OPT_HOST_PATH picks (0 auto, 1 copy, 2 direct or fail).  The call is
+ * ordered after earlier work on `stream`, and later work on `stream` sees
+ * its results. */
 int dpdr_allreduce_host(dpdr_plan_t plan, const void* const* x_host,
                         void* const* y_host, void* const* x_dev,
                         void* const* y_dev, dpdr_stream_t stream);

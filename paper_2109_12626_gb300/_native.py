@@ -18,7 +18,7 @@ DPDR_OP_SUM, DPDR_OP_MATMUL = 0, 1
  DPDR_ERR_NOT_COOPERATIVE, DPDR_ERR_OOM) = range(6)
 (OPT_FUSED_MODE, OPT_WAIT_LIMIT_NS, OPT_SKIP_RANK, OPT_SCHED_THREADS,
  OPT_SCHED_RANKS_PER_CTA, OPT_BLOCKS, OPT_SPLIT_DEPTH, OPT_SCHED_SLICES,
- OPT_HOST_CHUNK_BYTES) = range(1, 10)
+ OPT_HOST_CHUNK_BYTES, OPT_HOST_PATH) = range(1, 11)
 
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libdpdr.so")
 
@@ -183,13 +183,13 @@ class Plan:
         return out
 
     def info(self) -> dict:
-        v = np.zeros(14, np.int64)
-        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), 14),
+        v = np.zeros(15, np.int64)
+        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), 15),
                "dpdr_plan_info")
         keys = ("p", "m", "b", "max_depth", "auto_mode", "sched_ctas",
                 "sched_ranks_per_cta", "scratch_bytes", "vector_path",
                 "split_depth", "split_subtrees", "split_group", "sched_slices",
-                "topology")
+                "topology", "host_path")
         return {k: int(x) for k, x in zip(keys, v)}
 
     def set(self, key: int, value: int) -> None:
@@ -209,11 +209,13 @@ class Plan:
                                              _ptr_array(ys), _stream(stream)),
                "dpdr_allreduce_schedule")
 
-    def allreduce_host(self, xh: Sequence, yh: Sequence, xd: Sequence,
-                       yd: Sequence, stream=None) -> None:
-        """Host buffers in and out, device buffers as staging."""
+    def allreduce_host(self, xh: Sequence, yh: Sequence, xd: Sequence | None = None,
+                       yd: Sequence | None = None, stream=None) -> None:
+        """Host buffers in and out (device buffers as staging when the GPU
+        cannot address the host buffers directly)."""
         _check(lib().dpdr_allreduce_host(self._h, _ptr_array(xh), _ptr_array(yh),
-                                         _ptr_array(xd), _ptr_array(yd),
+                                         _ptr_array(xd) if xd is not None else None,
+                                         _ptr_array(yd) if yd is not None else None,
                                          _stream(stream)), "dpdr_allreduce_host")
 
     def bind(self, xs: Sequence, ys: Sequence) -> "Bound":

@@ -177,18 +177,69 @@ static int pipe_prepare(Plan* P, void* const* x_dev, void* const* y_dev, bool ve
     return DPDR_OK;
 }
 
+// Device addresses for host buffers the GPU can load and store directly:
+// pinned (page-locked, mapped into the unified address space) memory, or
+// pageable memory on systems whose GPU walks the CPU page tables (Grace
+// with NVLink-C2C).  Resolved once per set of host arrays.
+static bool resolve_direct(Plan* P, const void* const* xh, void* const* yh)
+{
+    const int p = P->p;
+    bool same = P->direct_ok && int(P->direct_xh.size()) == p;
+    for (int i = 0; i < p && same; i++) same = P->direct_xh[i] == xh[i] && P->direct_yh[i] == yh[i];
+    if (same) return true;
+    int pageable = 0;
+    if (cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, P->device) != cudaSuccess)
+        pageable = 0;
+    std::vector<const void*> dx(p), dy(p);
+    for (int k = 0; k < 2 * p; k++) {
+        const void* hp = k < p ? xh[k] : yh[k - p];
+        cudaPointerAttributes at;
+        const void* dp = nullptr;
+        if (cudaPointerGetAttributes(&at, hp) == cudaSuccess) {
+            if (at.type == cudaMemoryTypeHost && at.devicePointer) dp = at.devicePointer;
+            else if (at.type == cudaMemoryTypeUnregistered && pageable) dp = hp;
+        } else {
+            cudaGetLastError();
+        }
+        if (!dp) {
+            P->direct_ok = false;
+            return false;
+        }
+        (k < p ? dx[k] : dy[k - p]) = dp;
+    }
+    P->direct_xh.assign(xh, xh + p);
+    P->direct_yh.assign(yh, yh + p);
+    P->direct_dx = dx;
+    P->direct_dy = dy;
+    P->direct_ok = true;
+    return true;
+}
+
 extern "C" int dpdr_allreduce_host(dpdr_plan_t h, const void* const* x_host,
                                    void* const* y_host, void* const* x_dev,
                                    void* const* y_dev, dpdr_stream_t stream)
 {
     Plan* P = reinterpret_cast<Plan*>(h);
     if (!P) return fail(DPDR_ERR_INVALID, "dpdr_allreduce_host: NULL plan");
-    if (!x_host || !y_host || !x_dev || !y_dev)
+    if (!x_host || !y_host)
         return fail(DPDR_ERR_INVALID, "dpdr_allreduce_host: NULL pointer array");
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     for (int i = 0; i < P->p; i++)
         if (!x_host[i] || !y_host[i]) return fail(DPDR_ERR_INVALID, "NULL host buffer");
     if (P->m == 0) return DPDR_OK;
+    // direct: the streaming layout loads the inputs from host memory and
+    // stores the result to host memory, both link directions at once
+    if (P->host_path != 1 && resolve_direct(P, x_host, y_host)) {
+        int rc = prepare(P, P->direct_dx.data(), P->direct_dy.data(), s);
+        if (rc) return rc;
+        P->last_host_path = 2;
+        return fused_launch_cols(P, P->d_x, P->d_y, P->m, P->last_vector_path != 0, s, 1);
+    }
+    if (P->host_path == 2)
+        return fail(DPDR_ERR_INVALID, "dpdr_allreduce_host: host buffers not addressable by the GPU");
+    if (!x_dev || !y_dev)
+        return fail(DPDR_ERR_INVALID, "dpdr_allreduce_host: device staging buffers needed");
+    P->last_host_path = 1;
     int vec = 0;
     int rc = check_buffers(P, reinterpret_cast<const void* const*>(x_dev),
                            reinterpret_cast<const void* const*>(y_dev), &vec);
@@ -215,7 +266,7 @@ extern "C" int dpdr_allreduce_host(dpdr_plan_t h, const void* const* x_host,
         if (e == cudaSuccess) e = cudaStreamWaitEvent(s, in, 0);
         if (e != cudaSuccess) return cuda_fail(e, "host to device copy");
         rc = fused_launch_cols(P, reinterpret_cast<const char* const*>(tab + size_t(c) * 2 * p),
-                               tab + (size_t(c) * 2 + 1) * p, mc, vec != 0, s);
+                               tab + (size_t(c) * 2 + 1) * p, mc, vec != 0, s, 0);
         if (rc) return rc;
         e = cudaEventRecord(out, s);
         if (e == cudaSuccess) e = cudaStreamWaitEvent(P->pipe_out, out, 0);

@@ -56,6 +56,8 @@ struct Plan {
     int sched_slices = 0;      // CTAs per rank (column slices), 0 = auto
     int split_depth = -1;      // cut depth of the split layout, -1 = auto
     int64_t host_chunk = int64_t(1) << 30;  // bytes of rank data per host-pipeline chunk
+    int host_path = 0;         // dpdr_allreduce_host: 0 auto, 1 copy pipeline, 2 direct
+    int last_host_path = 0;    // path the last dpdr_allreduce_host took (1 or 2)
 
     // device memory: one allocation carved into the tables below
     char* dmem = nullptr;
@@ -104,6 +106,10 @@ struct Plan {
     int64_t pipe_cols = 0;
     int pipe_chunks = 0;
     std::vector<const void*> pipe_xd, pipe_yd;
+    // device addresses of host buffers the GPU reads and writes directly
+    std::vector<const void*> direct_xh, direct_yh;   // host arrays they came from
+    std::vector<const void*> direct_dx, direct_dy;
+    bool direct_ok = false;
 
     // facts
     int last_vector_path = 0;
@@ -130,7 +136,7 @@ int stage_pointers(Plan* P, const void* const* x, const void* const* y,
 // launchers
 int fused_launch(Plan* P, cudaStream_t s);      // fused.cu
 int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t mc, bool vec,
-                      cudaStream_t s);             // fused.cu
+                      cudaStream_t s, int force_mode);  // fused.cu (0: plan's choice)
 int fused_auto_mode(const Plan* P);             // fused.cu
 int fused_split_prepare(Plan* P, bool force, int depth);  // fused.cu
 int schedule_launch(Plan* P, cudaStream_t s);   // schedule.cu

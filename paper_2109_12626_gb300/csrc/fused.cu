@@ -110,16 +110,16 @@ int fused_split_prepare(Plan* P, bool force, int depth)
 
 int fused_launch(Plan* P, cudaStream_t s)
 {
-    return fused_launch_cols(P, P->d_x, P->d_y, P->m, P->last_vector_path != 0, s);
+    return fused_launch_cols(P, P->d_x, P->d_y, P->m, P->last_vector_path != 0, s, 0);
 }
 
 // The fused kernel on mc columns, with device tables of rank pointers that
 // may point into the middle of the rank buffers (a column chunk).
 int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t mc, bool vec,
-                      cudaStream_t s)
+                      cudaStream_t s, int force_mode)
 {
     if (mc == 0) return DPDR_OK;
-    int mode = P->fused_mode ? P->fused_mode : fused_auto_mode(P);
+    int mode = force_mode ? force_mode : P->fused_mode ? P->fused_mode : fused_auto_mode(P);
     const int lg = tile_lg_wu(P);
     if (mode == 2 && lg < 0) return fail(DPDR_ERR_INVALID, "tile mode: p too large");
     if (mode == 3 && !P->split_ready) return fail(DPDR_ERR_INVALID, "split mode: p < 2");

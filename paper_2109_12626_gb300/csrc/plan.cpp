@@ -411,6 +411,10 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
         P->split_depth = int(v);
         return fused_split_prepare(P, true, P->split_depth);
     }
+    case DPDR_OPT_HOST_PATH:
+        if (v < 0 || v > 2) return fail(DPDR_ERR_INVALID, "host path: 0, 1 or 2");
+        P->host_path = int(v);
+        return DPDR_OK;
     case DPDR_OPT_HOST_CHUNK_BYTES:
         if (v < 4096) return fail(DPDR_ERR_INVALID, "host chunk below 4096 bytes");
         P->host_chunk = v;
@@ -441,7 +445,7 @@ extern "C" int dpdr_plan_info(dpdr_plan_t h, int64_t* info, int n)
                          P->sched_ctas, P->sched_ranks_per_cta,
                          int64_t(P->dmem_bytes + P->d_split_bytes), P->last_vector_path,
                          P->split_s, P->split_nseg, P->split_group,
-                         P->sched_slices_used, P->topo};
+                         P->sched_slices_used, P->topo, P->last_host_path};
     const int k = int(sizeof v / sizeof v[0]);
     for (int i = 0; i < n; i++) info[i] = i < k ? v[i] : 0;
     return DPDR_OK;

@@ -195,26 +195,57 @@ def test_repeated_calls_and_pointer_changes(pkg, orc):
 
 @pytest.mark.parametrize("kind,p,m,chunk", [("float32", 32, 10007, 0), ("float32", 32, 10007, 4096),
                                             ("int32", 1152, 3001, 65536), ("mat2x2u32", 7, 2049, 4096),
-                                            ("float32", 3, 257, 4096)])
+                                            ("float32", 3, 257, 4096), ("mat2x2f32", 36, 1001, 0)])
+@pytest.mark.parametrize("path", ["auto", "copy"])
+@pytest.mark.parametrize("pinned", [True, False])
 @pytest.mark.parametrize("in_place", [False, True])
-def test_host_buffers_end_to_end(pkg, orc, kind, p, m, chunk, in_place):
-    """dpdr_allreduce_host: pinned host inputs, column chunks pipelined
-    through copy-in, kernel and copy-out streams, pinned host outputs."""
+def test_host_buffers_end_to_end(pkg, orc, kind, p, m, chunk, path, pinned, in_place):
+    """dpdr_allreduce_host: host inputs and outputs.  "auto" runs the kernel
+    directly on the host buffers when the GPU can address them (pinned, or
+    pageable on a GPU that walks the CPU page tables), "copy" forces the
+    pipeline of chunked copies through device buffers."""
     x = host_inputs(kind, 31, p, m)
     want = _want(orc, x, kind)
     dev = torch.device("cuda:0")
-    xh = [torch.from_numpy(np.ascontiguousarray(x[i]).view(np.int32).reshape(-1).copy()).pin_memory()
+    xh = [torch.from_numpy(np.ascontiguousarray(x[i]).view(np.int32).reshape(-1).copy())
           for i in range(p)]
-    yh = [torch.full_like(t, -9).pin_memory() for t in xh]
+    yh = [torch.full_like(t, -9) for t in xh]
+    if pinned:
+        xh = [t.pin_memory() for t in xh]
+        yh = [t.pin_memory() for t in yh]
+    if in_place:
+        yh = xh
     xd = [torch.empty_like(t, device=dev) for t in xh]
     yd = xd if in_place else [torch.empty_like(t, device=dev) for t in xh]
     with pkg.Plan(p, m, kind, 0) as plan:
         if chunk:
             plan.set(pkg.OPT_HOST_CHUNK_BYTES, chunk)
+        if path == "copy":
+            plan.set(pkg.OPT_HOST_PATH, 1)
         for _ in range(2):
+            if in_place:  # the inputs are overwritten: restore them
+                for i in range(p):
+                    xh[i].copy_(torch.from_numpy(np.ascontiguousarray(x[i]).view(np.int32).reshape(-1)))
             plan.allreduce_host(xh, yh, xd, yd)
             plan.sync()
             _check_all(yh, want)
+        took = plan.info()["host_path"]
+        assert took == (1 if path == "copy" else took)
+        if path == "auto" and pinned:
+            assert took == 2  # pinned memory is always addressable
+
+
+def test_host_buffers_direct_needs_no_device_buffers(pkg, orc):
+    kind, p, m = "float32", 32, 4099
+    x = host_inputs(kind, 33, p, m)
+    want = _want(orc, x, kind)
+    xh = [torch.from_numpy(x[i].copy()).pin_memory() for i in range(p)]
+    yh = [torch.zeros(m).pin_memory() for _ in range(p)]
+    with pkg.Plan(p, m, kind, 0) as plan:
+        plan.allreduce_host(xh, yh)
+        plan.sync()
+        assert plan.info()["host_path"] == 2
+    _check_all(yh, want)
 
 
 def test_invalid_arguments(pkg):
