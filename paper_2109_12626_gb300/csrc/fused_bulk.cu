@@ -195,8 +195,8 @@ fused_bulk_kernel(FusedArgs a)
     for (int64_t u = u_first + int64_t(blockIdx.x) * kBulkConsumers + tid; u < a.nvec; u += stride)
         stream_column<VecUnit<Op>>(a, u, slot, kBulkConsumers);
     for (int64_t e = int64_t(blockIdx.x) * kBulkConsumers + tid; e < a.nscalar; e += stride)
-        stream_column<OneUnit<Op>>(a, a.scalar_base + e, reinterpret_cast<Elem<Op>*>(slots) + tid,
-                                   kBulkConsumers);
+        stream_column<OneUnit<Op>>(a, a.scalar_base + e, one_slots<Op>(slots, tid),
+                                   one_slot_stride<Op>(kBulkConsumers));
 }
 
 

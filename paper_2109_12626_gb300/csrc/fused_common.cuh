@@ -156,6 +156,21 @@ __device__ __forceinline__ void stream_column(const FusedArgs& a, int64_t u,
     for (int i = 0; i < p; i++) U::st(rank_ptr_w(a.y, i), u, y);
 }
 
+// The depth slots of thread t sit in 16-byte cells t, t + n, t + 2n, ... of
+// a [depth][n] array of uint4 (n threads).  A thread folding single elements
+// keeps its slots in the same cells (an element is at most 16 bytes), so its
+// slots never overlap another thread's, whatever unit each thread folds.
+template <class Op>
+__device__ __forceinline__ Elem<Op>* one_slots(uint4* cells, int t)
+{
+    return reinterpret_cast<Elem<Op>*>(cells + t);
+}
+template <class Op>
+__device__ __forceinline__ int one_slot_stride(int n)
+{
+    return n * int(sizeof(uint4) / sizeof(Elem<Op>));
+}
+
 // launchers, one per layout (dispatch on the plan's element type)
 int launch_stream(Plan* P, FusedArgs a, cudaStream_t s);
 int launch_tile(Plan* P, FusedArgs a, cudaStream_t s);

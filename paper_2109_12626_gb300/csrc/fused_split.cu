@@ -80,9 +80,9 @@ fused_split_reduce_kernel(FusedArgs a)
     if (u < a.nvec) {
         split_reduce_column<VecUnit<Op>>(a, blockIdx.y, u, smem + threadIdx.x, blockDim.x);
     } else if (u < a.nvec + a.nscalar) {
-        auto* slot = reinterpret_cast<Elem<Op>*>(smem) + threadIdx.x;
-        split_reduce_column<OneUnit<Op>>(a, blockIdx.y, a.scalar_base + (u - a.nvec), slot,
-                                         blockDim.x);
+        split_reduce_column<OneUnit<Op>>(a, blockIdx.y, a.scalar_base + (u - a.nvec),
+                                         one_slots<Op>(smem, threadIdx.x),
+                                         one_slot_stride<Op>(blockDim.x));
     }
 }
 
@@ -95,9 +95,9 @@ fused_split_finish_kernel(FusedArgs a)
     if (u < a.nvec) {
         split_finish_column<VecUnit<Op>>(a, blockIdx.y, u, smem + threadIdx.x, blockDim.x);
     } else if (u < a.nvec + a.nscalar) {
-        auto* slot = reinterpret_cast<Elem<Op>*>(smem) + threadIdx.x;
-        split_finish_column<OneUnit<Op>>(a, blockIdx.y, a.scalar_base + (u - a.nvec), slot,
-                                         blockDim.x);
+        split_finish_column<OneUnit<Op>>(a, blockIdx.y, a.scalar_base + (u - a.nvec),
+                                         one_slots<Op>(smem, threadIdx.x),
+                                         one_slot_stride<Op>(blockDim.x));
     }
 }
 

@@ -17,8 +17,8 @@ fused_stream_kernel(FusedArgs a)
     if (u < a.nvec) {
         stream_column<VecUnit<Op>>(a, u, smem + threadIdx.x, blockDim.x);
     } else if (u < a.nvec + a.nscalar) {
-        auto* slot = reinterpret_cast<Elem<Op>*>(smem) + threadIdx.x;
-        stream_column<OneUnit<Op>>(a, a.scalar_base + (u - a.nvec), slot, blockDim.x);
+        stream_column<OneUnit<Op>>(a, a.scalar_base + (u - a.nvec), one_slots<Op>(smem, threadIdx.x),
+                                   one_slot_stride<Op>(blockDim.x));
     }
 }
 

@@ -34,6 +34,11 @@ CASES = [
     ("p36_m65536_matf", "mat2x2f32", 6, 36, 65536, {}, [16, 1, 7]),
     ("p1152_m1025_matf", "mat2x2f32", 6, 1152, 1025, {}, [1, 4]),
     ("p3_m9_matf", "mat2x2f32", 6, 3, 9, {}, [1, 9]),
+    # ragged tails whose single-element thread sits in another warp than the
+    # vector threads of its block (their shared-memory slots must not meet)
+    ("p3_m801_f32", "float32", 9, 3, 801, {}, [2]),
+    ("p32_m803_int32", "int32", 9, 32, 803, {}, [3]),
+    ("p1152_m1021_f32", "float32", 9, 1152, 1021, {}, [2]),
 ]
 
 
