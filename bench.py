@@ -363,14 +363,16 @@ def run_sweep(args, w) -> int:
     p, kind, es = w["p"], w["kind"], ESIZE[w["kind"]]
     if args.sweep == "m":
         top = int(args.m or (1 << 23)).bit_length() - 1
-        for k in range(0, top + 1):
-            m = 1 << k
+        ms = ([int(v) for v in args.mlist.split(",")] if args.mlist
+              else [1 << k for k in range(0, top + 1)])
+        for m in ms:
             ww = dict(w, m=m)
             xs = gen_device_inputs(ww, dev)
             ys = [torch.empty_like(x) for x in xs]
             rec = {"sweep": "m", "workload": args.workload, "p": p, "m": m,
                    "topology": args.topology}
-            with pkg.Plan(p, m, kind, 0, topology=args.topology) as plan:
+            b0 = -(-m // args.block_size) if args.block_size else 0
+            with pkg.Plan(p, m, kind, b0, topology=args.topology) as plan:
                 bd = plan.bind(xs, ys)
                 t = _timed(lambda: bd.allreduce(), 20, None, graph=True)
                 info = plan.info()
@@ -439,6 +441,9 @@ def main(argv=None) -> int:
     ap.add_argument("--topology", choices=("dual", "single"), default="dual",
                     help="dual roots (the paper's method) or one tree (Sec. 1.2 variant)")
     ap.add_argument("--p", type=int, default=None, help="override p (sweeps)")
+    ap.add_argument("--block-size", type=int, default=None,
+                    help="schedule kernel blocks of this many elements: b = ceil(m / size)")
+    ap.add_argument("--mlist", default=None, help="comma-separated m values for --sweep m")
     ap.add_argument("--host-path", type=int, default=0,
                     help="e2e leg: 0 direct when possible, 1 copy pipeline, 2 direct")
     args = ap.parse_args(argv)
@@ -472,6 +477,8 @@ def main(argv=None) -> int:
     p, m, kind = w["p"], w["m"], w["kind"]
     es = ESIZE[kind]
     b = args.b if args.b is not None else (w.get("b") or 0)
+    if args.block_size:
+        b = -(-m // args.block_size)
     xs = gen_device_inputs(w, dev)
     ys = [torch.empty_like(x) for x in xs]
     plan = pkg.Plan(p, m, kind, b, topology=args.topology)
