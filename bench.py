@@ -352,8 +352,9 @@ def _timed(fn, reps, stream, graph=False):
 
 def run_sweep(args, w) -> int:
     """--sweep m: every m = 2^0 .. 2^k of the workload, fused kernel (its
-    automatic layout, CUDA-graph replay so launch overhead is excluded) and
-    schedule kernel at the block-count rule.  --sweep b: the schedule
+    automatic layout) and schedule kernel (its automatic transport) at the
+    block-count rule, both timed as CUDA-graph replays so host launch
+    overhead is excluded.  --sweep b: the schedule
     kernel's time against b at one m, with the Sec. 1.2 cost model fitted.
     One JSON line per point, then a summary line."""
     import torch
@@ -379,11 +380,14 @@ def run_sweep(args, w) -> int:
                 rec["fused"] = {"us": round(t * 1e6, 2), "gbs": round(2 * p * m * es / t / 1e9, 2),
                                 "layout": LAYOUTS[info["auto_mode"]],
                                 "split_depth": info["split_depth"] if info["auto_mode"] == 3 else None}
-                t = _timed(lambda: bd.allreduce_schedule(), 3 if m >= (1 << 20) else 10, None)
+                t = _timed(lambda: bd.allreduce_schedule(), 3 if m >= (1 << 20) else 10, None,
+                           graph=True)
                 plan.sync()
                 rec["schedule"] = {"b": info["b"], "us": round(t * 1e6, 2),
                                    "gbs": round(2 * p * m * es / t / 1e9, 2),
-                                   "slices": plan.info()["sched_slices"]}
+                                   "slices": plan.info()["sched_slices"],
+                                   "transport": ("counters", "words")[
+                                       info["sched_transport"] - 1]}
             print(json.dumps(rec), flush=True)
             del xs, ys
             torch.cuda.empty_cache()
@@ -397,7 +401,8 @@ def run_sweep(args, w) -> int:
     for b in bs:
         with pkg.Plan(p, m, kind, b, topology=args.topology) as plan:
             bd = plan.bind(xs, ys)
-            t = _timed(lambda: bd.allreduce_schedule(), 5 if m >= (1 << 20) else 10, None)
+            t = _timed(lambda: bd.allreduce_schedule(), 5 if m >= (1 << 20) else 10, None,
+                       graph=True)
             plan.sync()
             points.append((b, t))
             print(json.dumps({"sweep": "b", "workload": args.workload, "topology": args.topology,

@@ -122,7 +122,8 @@ int dpdr_block_count_rule(int p, int64_t m, double kappa);
 /* Builds the trees, the block partition and the device tables for p ranks
  * of m elements of (dtype, op) on the current CUDA device, and allocates the
  * plan's device scratch (rank-pointer tables, handshake counters, the dual
- * roots' exchange slots, an error word).  b is the number of pipeline
+ * roots' exchange slots, an error word, and the word arrays of the
+ * schedule kernel's flagged-word transport when it is selected).  b is the number of pipeline
  * blocks (Algorithm 1); b == 0 selects dpdr_block_count_rule(p, m, 0);
  * b is clamped to [1, max(m,1)].  p >= 1, m >= 0.  Returns NULL on error
  * (see dpdr_last_error).  Not thread-safe with respect to one plan. */
@@ -166,7 +167,19 @@ int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
  *                             dpdr_allreduce_host's copy pipeline (default
  *                             2^30, minimum 4096)
  *   DPDR_OPT_HOST_PATH        dpdr_allreduce_host: 0 direct when possible,
- *                             else copy; 1 copy pipeline; 2 direct only */
+ *                             else copy; 1 copy pipeline; 2 direct only
+ *   DPDR_OPT_SCHED_TRANSPORT  how dpdr_allreduce_schedule moves a block
+ *                             between virtual ranks (same rounds, steps and
+ *                             result either way): 1 counters -- the block is
+ *                             written, then a release/acquire counter
+ *                             publishes it; 2 flagged words -- every 32-bit
+ *                             word travels with the call's epoch in one
+ *                             64-bit store and the receiver polls the words,
+ *                             which halves the latency of short blocks but
+ *                             keeps 4 p m esize bytes of word arrays on the
+ *                             device; 0 (default) chooses 2 while
+ *                             m * esize <= 32 KiB and those arrays stay
+ *                             within 1 GiB, else 1 */
 enum {
     DPDR_OPT_FUSED_MODE = 1,
     DPDR_OPT_WAIT_LIMIT_NS = 2,
@@ -177,7 +190,8 @@ enum {
     DPDR_OPT_SPLIT_DEPTH = 7,
     DPDR_OPT_SCHED_SLICES = 8,
     DPDR_OPT_HOST_CHUNK_BYTES = 9,
-    DPDR_OPT_HOST_PATH = 10
+    DPDR_OPT_HOST_PATH = 10,
+    DPDR_OPT_SCHED_TRANSPORT = 11
 };
 int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
 
@@ -190,7 +204,8 @@ int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
  *   group of its second kernel (0 when the split layout is not prepared)
  *   [12] CTAs per rank (column slices) of the schedule kernel
  *   [13] topology (dpdr_topology)
- *   [14] path of the last dpdr_allreduce_host: 1 copy pipeline, 2 direct */
+ *   [14] path of the last dpdr_allreduce_host: 1 copy pipeline, 2 direct
+ *   [15] transport of dpdr_allreduce_schedule: 1 counters, 2 flagged words */
 int dpdr_plan_info(dpdr_plan_t plan, int64_t* info, int n);
 
 /* Releases the plan's device and host memory.  The caller must first make
@@ -210,8 +225,10 @@ int dpdr_allreduce(dpdr_plan_t plan, const void* const* x, void* const* y,
 /* Schedule-faithful kernel: runs Algorithm 1 for every virtual rank, rounds
  * j = 0..b+d_i, each round's exchanges with child_0, child_1 and the parent
  * or dual, as one cooperative persistent launch in which CTAs own ranks and
- * exchange pipeline blocks through device memory with release/acquire
- * counters.  Same result as dpdr_allreduce.  Every wait is bounded
+ * exchange pipeline blocks through device memory, published either by
+ * release/acquire counters or as epoch-flagged words
+ * (DPDR_OPT_SCHED_TRANSPORT).  Same result as dpdr_allreduce.  Two calls
+ * on one plan that overlap on the GPU (two streams) race on its scratch.  Every wait is bounded
  * (DPDR_OPT_WAIT_LIMIT_NS); an expired wait ends the kernel early and is
  * reported as DPDR_ERR_TIMEOUT by dpdr_plan_sync.  Returns
  * DPDR_ERR_NOT_COOPERATIVE if the ranks cannot be co-resident.

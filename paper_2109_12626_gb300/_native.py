@@ -18,7 +18,7 @@ DPDR_OP_SUM, DPDR_OP_MATMUL = 0, 1
  DPDR_ERR_NOT_COOPERATIVE, DPDR_ERR_OOM) = range(6)
 (OPT_FUSED_MODE, OPT_WAIT_LIMIT_NS, OPT_SKIP_RANK, OPT_SCHED_THREADS,
  OPT_SCHED_RANKS_PER_CTA, OPT_BLOCKS, OPT_SPLIT_DEPTH, OPT_SCHED_SLICES,
- OPT_HOST_CHUNK_BYTES, OPT_HOST_PATH) = range(1, 11)
+ OPT_HOST_CHUNK_BYTES, OPT_HOST_PATH, OPT_SCHED_TRANSPORT) = range(1, 12)
 
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libdpdr.so")
 
@@ -183,13 +183,13 @@ class Plan:
         return out
 
     def info(self) -> dict:
-        v = np.zeros(15, np.int64)
-        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), 15),
+        v = np.zeros(16, np.int64)
+        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), 16),
                "dpdr_plan_info")
         keys = ("p", "m", "b", "max_depth", "auto_mode", "sched_ctas",
                 "sched_ranks_per_cta", "scratch_bytes", "vector_path",
                 "split_depth", "split_subtrees", "split_group", "sched_slices",
-                "topology", "host_path")
+                "topology", "host_path", "sched_transport")
         return {k: int(x) for k, x in zip(keys, v)}
 
     def set(self, key: int, value: int) -> None:

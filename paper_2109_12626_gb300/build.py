@@ -22,7 +22,8 @@ LIB = os.path.join(HERE, "libdpdr.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 SOURCES = ["plan.cpp", "api.cpp", "fused.cu", "fused_stream.cu", "fused_tile.cu",
-           "fused_split.cu", "fused_bulk.cu", "schedule.cu"]
+           "fused_split.cu", "fused_bulk.cu", "schedule.cu",
+           "schedule_ll.cu"]
 
 
 def nvcc() -> str:

@@ -121,7 +121,7 @@ extern "C" int dpdr_allreduce_schedule(dpdr_plan_t h, const void* const* x,
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     int rc = prepare(P, x, reinterpret_cast<const void* const*>(y), s);
     if (rc) return rc;
-    return schedule_launch(P, s);
+    return schedule_transport(P) == 2 ? schedule_ll_launch(P, s) : schedule_launch(P, s);
 }
 
 // Column chunks of about host_chunk bytes of rank data (default 1 GB), each

@@ -55,6 +55,7 @@ struct Plan {
     int sched_rpc = 0;         // ranks per CTA, 0 = auto
     int sched_slices = 0;      // CTAs per rank (column slices), 0 = auto
     int split_depth = -1;      // cut depth of the split layout, -1 = auto
+    int sched_transport = 0;   // schedule kernel: 0 auto, 1 counters, 2 flagged words
     int64_t host_chunk = int64_t(1) << 30;  // bytes of rank data per host-pipeline chunk
     int host_path = 0;         // dpdr_allreduce_host: 0 auto, 1 copy pipeline, 2 direct
     int last_host_path = 0;    // path the last dpdr_allreduce_host took (1 or 2)
@@ -75,6 +76,10 @@ struct Plan {
     int* d_cta_first = nullptr;      // schedule chunk -> first rank (+1 entry)
     char* d_sched = nullptr;         // own allocation: counters + chunk table
     size_t d_sched_bytes = 0;
+    // low-latency transport of the schedule kernel (schedule_ll.cu): control
+    // words, then the up and down word arrays; own allocation
+    char* d_ll = nullptr;
+    size_t d_ll_bytes = 0;
 
     // rank-pointer staging (pinned host), copied to d_x / d_y when they change
     const void** h_ptrs = nullptr;   // [2p]
@@ -141,5 +146,11 @@ int fused_auto_mode(const Plan* P);             // fused.cu
 int fused_split_prepare(Plan* P, bool force, int depth);  // fused.cu
 int schedule_launch(Plan* P, cudaStream_t s);   // schedule.cu
 int schedule_configure(Plan* P);                // schedule.cu
+int schedule_transport(const Plan* P);          // schedule_ll.cu: 1 counters, 2 words
+const void* schedule_ll_kernel_for(int dtype);  // schedule_ll.cu
+size_t schedule_ll_bytes(const Plan* P);        // schedule_ll.cu
+int64_t schedule_ll_slice_elems(const Plan* P); // schedule_ll.cu
+int schedule_ll_prepare(Plan* P);               // schedule_ll.cu
+int schedule_ll_launch(Plan* P, cudaStream_t s);  // schedule_ll.cu
 
 }  // namespace dpdr

@@ -13,17 +13,32 @@ using fused::tile_lg_wu;
 static int64_t stream_target(const Plan* P) { return int64_t(P->num_sms) * 1024; }
 
 // Layout choice, from layout sweeps measured on GB300:
-//  * deep trees (p >= 128) with at least 4096 column units: the split layout,
-//    whose read phase (first kernel) and write phase (second kernel) keep
-//    HBM traffic one-directional; at p = 1152 it beats the tile from
-//    m = 2^14 and column streaming up to the largest sizes;
+//  * deep trees (p >= 128) whose p input rows total at most kTileMaxBytes:
+//    the shared-memory tile, the layout with the lowest fixed cost (p = 288,
+//    m = 2^15 int32: 22.6 us against the split layout's 27.3 us; at 75.5 MB,
+//    twice that, the split layout wins at p = 288, 576 and 1152);
+//  * deep trees (p >= kSplitMinRanks) above that: the split layout, whose
+//    read phase (first kernel) and write phase (second kernel) keep HBM
+//    traffic one-directional; at p = 1152 it beats column streaming up to
+//    the largest sizes;
 //  * otherwise column streaming once there are a quarter of the columns it
 //    needs to fill the GPU (p = 36, 2x2 matrices, m = 2^16: 13 us against the
 //    tile's 15 us), and the shared-memory tile below that.
+constexpr int64_t kTileMaxBytes = int64_t(40) << 20;
+constexpr int kSplitMinRanks = 128;
+constexpr int64_t kSplitWork = int64_t(1) << 17;
+
+static bool tile_preferred(const Plan* P)
+{
+    return P->p >= 128 && tile_lg_wu(P) >= 0 &&
+           int64_t(P->p) * P->m * P->esize <= kTileMaxBytes;
+}
+
 int fused_auto_mode(const Plan* P)
 {
     const int64_t units = P->m * int64_t(P->esize) / 16;
-    if (P->p >= 128 && units >= 4096 && P->split_ready) return 3;
+    if (tile_preferred(P)) return 2;
+    if (P->p >= kSplitMinRanks && units >= 4096 && P->split_ready) return 3;
     if (units >= stream_target(P) / 4) return 1;
     if (tile_lg_wu(P) >= 0) return 2;
     return P->split_ready ? 3 : 1;
@@ -34,7 +49,7 @@ int fused_auto_mode(const Plan* P)
 static bool split_wanted(const Plan* P)
 {
     const int64_t units = P->m * int64_t(P->esize) / 16;
-    return P->p >= 128 && units >= 4096;
+    return P->p >= kSplitMinRanks && units >= 4096 && !tile_preferred(P);
 }
 
 // Split layout: cut depth s, subtree table, top-of-tree item list, rank
@@ -46,19 +61,20 @@ int fused_split_prepare(Plan* P, bool force, int depth)
     const int p = P->p;
     if (p < 2) return DPDR_OK;  // one rank: nothing to split
     const int64_t units = std::max<int64_t>(1, P->m * int64_t(P->esize) / 16);
-    const int64_t target = stream_target(P);
-    // automatic cut, from the measured best cuts at p = 1152 (the first
-    // kernel wants many subtree columns, the second kernel's sequential walk
-    // over the 2^(s+2) - 2 rows grows with s): depth 4 below 16 K column
-    // units, 3 below 64 K, 2 below 256 K, 1 below 512 K, 0 above; never
-    // deeper than the tree allows
+    // automatic cut: the shallowest depth whose subtrees (2^s per tree) times
+    // the column units give the first kernel kSplitWork independent walks;
+    // a deeper cut only lengthens the second kernel's walk over the
+    // 2^(s+2) - 2 rows.  Measured at p = 128 ... 1152, int32, m = 2^14 ...
+    // 2^22: within 2 % of the best cut everywhere (at m = 2^17 the cut at
+    // depth 1 takes 28.9 us at p = 128 where depth 3 took 39.5 us); never
+    // deeper than 4 or than the tree allows
     int s = depth;
     if (s < 0) {
-        s = units < (16 << 10) ? 4 : units < (64 << 10) ? 3 : units < (256 << 10) ? 2
-          : units < (512 << 10) ? 1 : 0;
+        const int64_t trees = P->r0 >= 0 ? 2 : 1;
+        s = 0;
+        while (s < 4 && (trees << s) * units < kSplitWork) s++;
         s = std::min(s, std::max(0, P->max_depth - 2));
     }
-    (void)target;
     s = std::min(s, P->max_depth);
     if (P->split_ready && P->split_s == s) return DPDR_OK;
     if (!force && !split_wanted(P)) return DPDR_OK;
@@ -80,6 +96,7 @@ int fused_split_prepare(Plan* P, bool force, int depth)
         P->d_split_bytes = 0;
         P->split_ready = false;
     }
+    const int64_t target = stream_target(P);
     int64_t groups = std::min<int64_t>(p, std::max<int64_t>(1, (target + units - 1) / units));
     P->split_group = int((p + groups - 1) / groups);
     P->split_s = s;

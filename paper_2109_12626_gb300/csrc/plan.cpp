@@ -223,6 +223,7 @@ static void free_plan(Plan* P)
     if (P->d_pipe) cudaFree(P->d_pipe);
     if (P->d_split) cudaFree(P->d_split);
     if (P->d_sched) cudaFree(P->d_sched);
+    if (P->d_ll) cudaFree(P->d_ll);
     if (P->h_ptrs) cudaFreeHost(P->h_ptrs);
     if (P->dmem) cudaFree(P->dmem);
     delete P;
@@ -348,6 +349,7 @@ extern "C" dpdr_plan_t dpdr_plan_topo(int p, int64_t m, dpdr_dtype dtype, dpdr_o
         return nullptr;
     }
     if (allocate(P) != DPDR_OK || schedule_configure(P) != DPDR_OK ||
+        (schedule_transport(P) == 2 && schedule_ll_prepare(P) != DPDR_OK) ||
         fused_split_prepare(P, false, P->split_depth) != DPDR_OK) {
         free_plan(P);
         return nullptr;
@@ -411,6 +413,19 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
         P->split_depth = int(v);
         return fused_split_prepare(P, true, P->split_depth);
     }
+    case DPDR_OPT_SCHED_TRANSPORT: {
+        if (v < 0 || v > 2) return fail(DPDR_ERR_INVALID, "schedule transport: 0, 1 or 2");
+        const int was = P->sched_transport;
+        P->sched_transport = int(v);
+        if (schedule_transport(P) == 2) {
+            const int rc = schedule_ll_prepare(P);
+            if (rc) {
+                P->sched_transport = was;
+                return rc;
+            }
+        }
+        return schedule_configure(P);
+    }
     case DPDR_OPT_HOST_PATH:
         if (v < 0 || v > 2) return fail(DPDR_ERR_INVALID, "host path: 0, 1 or 2");
         P->host_path = int(v);
@@ -443,9 +458,11 @@ extern "C" int dpdr_plan_info(dpdr_plan_t h, int64_t* info, int n)
     if (!P || !info) return fail(DPDR_ERR_INVALID, "dpdr_plan_info: NULL");
     const int64_t v[] = {P->p, P->m, P->b, P->max_depth, fused_auto_mode(P),
                          P->sched_ctas, P->sched_ranks_per_cta,
-                         int64_t(P->dmem_bytes + P->d_split_bytes), P->last_vector_path,
-                         P->split_s, P->split_nseg, P->split_group,
-                         P->sched_slices_used, P->topo, P->last_host_path};
+                         int64_t(P->dmem_bytes + P->d_split_bytes + P->d_sched_bytes +
+                                 P->d_ll_bytes),
+                         P->last_vector_path, P->split_s, P->split_nseg, P->split_group,
+                         P->sched_slices_used, P->topo, P->last_host_path,
+                         schedule_transport(P)};
     const int k = int(sizeof v / sizeof v[0]);
     for (int i = 0; i < n; i++) info[i] = i < k ? v[i] : 0;
     return DPDR_OK;

@@ -40,13 +40,12 @@
 #include <algorithm>
 #include <mutex>
 
-#include "dpdr_internal.h"
-#include "ops.cuh"
+#include "schedule_common.cuh"
 
 namespace dpdr {
 namespace {
 
-constexpr int kSchedMaxThreads = 256;
+constexpr int kSchedMaxThreads = sched::kMaxThreads;
 
 struct SchedArgs {
     const char* const* x;
@@ -71,32 +70,16 @@ struct SchedArgs {
     int nchunks;   // rank ranges (CTA index = slice * nchunks + chunk)
 };
 
-__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p)
-{
-    uint32_t v;
-    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
-__device__ __forceinline__ void st_release(uint32_t* p, uint32_t v)
-{
-    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-__device__ __forceinline__ uint32_t ld_relaxed(const uint32_t* p)
-{
-    uint32_t v;
-    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
-__device__ __forceinline__ uint64_t now_ns()
-{
-    uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
+using sched::ld_acquire;
+using sched::ld_relaxed;
+using sched::now_ns;
+using sched::rank_in;
+using sched::rank_out;
+using sched::st_release;
 
 __device__ __forceinline__ int64_t blk_start(const SchedArgs& a, int j)
 {
-    return int64_t(j) * a.q + lmin(j, a.rem);
+    return sched::block_start(a.q, a.rem, j);
 }
 
 // Start of column slice g (of nslices) of the element range [s, e): even
@@ -104,10 +87,7 @@ __device__ __forceinline__ int64_t blk_start(const SchedArgs& a, int j)
 template <int EPV>
 __device__ __forceinline__ int64_t slice_at(const SchedArgs& a, int64_t s, int64_t e, int g)
 {
-    if (g <= 0) return s;
-    if (g >= a.nslices) return e;
-    const int64_t b = (s + (e - s) * g / a.nslices) / EPV * EPV;
-    return b < s ? s : b;
+    return sched::slice_bound<EPV>(s, e, g, a.nslices);
 }
 
 // Thread 0 waits for *ctr >= target within the plan's time bound; the CTA
@@ -227,8 +207,8 @@ __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j, int 
     const int d = __ldg(a.depth + i);
     const int c0 = __ldg(a.child0 + i), c1 = __ldg(a.child1 + i);
     const int par = __ldg(a.parent + i);
-    const char* xi = reinterpret_cast<const char*>(__ldg(reinterpret_cast<const unsigned long long*>(a.x) + i));
-    char* yi = reinterpret_cast<char*>(__ldg(reinterpret_cast<const unsigned long long*>(a.y) + i));
+    const char* xi = rank_in(a.x, i);
+    char* yi = rank_out(a.y, i);
     const bool root = par < 0;
     const bool paired_root = root && a.r0 >= 0;
     const bool inb = j < a.b;
@@ -246,8 +226,8 @@ __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j, int 
         if (!cta_wait(a, up + c, uint32_t(j + 1), i, j, k)) return false;
         const bool leaf = __ldg(a.child0 + c) < 0;
         const char* src = leaf
-            ? reinterpret_cast<const char*>(__ldg(reinterpret_cast<const unsigned long long*>(a.x) + c))
-            : reinterpret_cast<const char*>(__ldg(reinterpret_cast<const unsigned long long*>(a.y) + c));
+            ? rank_in(a.x, c)
+            : rank_in(a.y, c);
         block_op<Op>(a, dst, src, have ? dst : xi, s, e);  // Y[j] = t (.) Y[j]
         have = true;
         __syncthreads();
@@ -285,7 +265,7 @@ __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j, int 
     const int kf = j - d;
     if (kf >= 0 && kf < a.b) {
         if (!cta_wait(a, down + par, uint32_t(kf + 1), i, j, 3)) return false;
-        const char* yp = reinterpret_cast<const char*>(__ldg(reinterpret_cast<const unsigned long long*>(a.y) + par));
+        const char* yp = rank_in(a.y, par);
         const int64_t ks = blk_start(a, kf), ke = blk_start(a, kf + 1);
         block_op<Op>(a, yi, nullptr, yp, slice_at<EPV>(a, ks, ke, g), slice_at<EPV>(a, ks, ke, g + 1));
         publish(a, down + i, uint32_t(kf + 1), i);
@@ -330,14 +310,20 @@ const void* kernel_for(int dtype)
 // Choose the CTA layout so that every CTA can be resident at once: ranks per
 // CTA (rank ranges never straddle the trees) and, when the GPU has room for
 // more CTAs than ranks, CTAs per rank (column slices of at least 1024
-// elements).  Allocates the counters for that many slices and uploads the
+// elements with counters, one word batch per thread with flagged words).
+// Allocates the counters for that many slices and uploads the
 // chunk -> first rank table.
 int schedule_configure(Plan* P)
 {
-    int occ = 0;
+    // one layout serves both transports: CTAs that fit for either kernel
+    int occ = 0, occ_ll = 0;
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
         &occ, kernel_for(P->dtype), P->sched_threads, 0);
+    if (e == cudaSuccess)
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+            &occ_ll, schedule_ll_kernel_for(P->dtype), P->sched_threads, 0);
     if (e != cudaSuccess) return cuda_fail(e, "schedule occupancy");
+    occ = std::min(occ, occ_ll);
     const int64_t kmax = int64_t(occ) * P->num_sms;
     // rank chunks never straddle the two trees (one tree: n0 = 0)
     const int n0 = P->r0 >= 0 ? P->p / 2 : 0, n1 = P->p - n0;
@@ -356,9 +342,14 @@ int schedule_configure(Plan* P)
     const int nchunks = int(first.size()) - 1;
     int G = P->sched_slices;
     if (G == 0) {
+        // counters: slices of at least 1024 elements; flagged words: one
+        // batch of words per thread
         const int64_t blk = (P->m + P->b - 1) / std::max(P->b, 1);
         const int64_t room = std::max<int64_t>(1, kmax / nchunks);
-        G = int(std::max<int64_t>(1, std::min<int64_t>({room, blk / 1024, 64})));
+        const int64_t want = schedule_transport(P) == 2
+            ? (blk + schedule_ll_slice_elems(P) - 1) / schedule_ll_slice_elems(P)
+            : blk / 1024;
+        G = int(std::max<int64_t>(1, std::min<int64_t>({room, want, 64})));
     }
     const size_t words = 2 * size_t(P->p) * G + 1;
     const size_t bytes = (words * sizeof(uint32_t) + 255) / 256 * 256 + sizeof(int) * first.size();

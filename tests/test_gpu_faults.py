@@ -24,7 +24,8 @@ def pkg():
 
 
 @pytest.mark.parametrize("p,skip", [(7, 0), (7, 6), (36, 17), (1152, 700)])
-def test_silent_rank_times_out_and_recovers(pkg, orc, p, skip):
+@pytest.mark.parametrize("transport", [1, 2], ids=["counters", "words"])
+def test_silent_rank_times_out_and_recovers(pkg, orc, p, skip, transport):
     from paper_2109_12626_gb300 import DpdrError
     kind, m = "int32", 1000
     x = host_inputs(kind, 41, p, m, lo=-1000, hi=1000)
@@ -33,6 +34,7 @@ def test_silent_rank_times_out_and_recovers(pkg, orc, p, skip):
     with pkg.Plan(p, m, kind, 4) as plan:
         plan.set(pkg.OPT_WAIT_LIMIT_NS, 20_000_000)   # 20 ms
         plan.set(pkg.OPT_SKIP_RANK, skip)
+        plan.set(pkg.OPT_SCHED_TRANSPORT, transport)
         ys, _ = empty_like_ranks(xs)
         plan.allreduce_schedule(xs, ys)
         with pytest.raises(DpdrError) as e:

@@ -85,8 +85,12 @@ def test_fused_matches_oracle(pkg, orc, case, mode):
         assert np.array_equal(bits(xs[i]), expect_bits(x[i]))
 
 
+TRANSPORTS = {"counters": 1, "words": 2}
+
+
 @pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
-def test_schedule_matches_oracle(pkg, orc, case):
+@pytest.mark.parametrize("transport", list(TRANSPORTS))
+def test_schedule_matches_oracle(pkg, orc, case, transport):
     _, kind, seed, p, m, kw, blist = case
     dev = torch.device("cuda:0")
     x = host_inputs(kind, seed, p, m, **kw)
@@ -95,6 +99,8 @@ def test_schedule_matches_oracle(pkg, orc, case):
     for b in blist:
         ys, _ = empty_like_ranks(xs)
         with pkg.Plan(p, m, kind, b) as plan:
+            plan.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[transport])
+            assert plan.info()["sched_transport"] == TRANSPORTS[transport]
             plan.allreduce_schedule(xs, ys)
             plan.sync()
         _check_all(ys, want)
@@ -103,11 +109,13 @@ def test_schedule_matches_oracle(pkg, orc, case):
 
 
 FUSED_RUNS = {"fused_stream": 1, "fused_tile": 2, "fused_split": 3, "fused_bulk": 4}
-RUNS = list(FUSED_RUNS) + ["schedule"]
+SCHED_RUNS = {"schedule_counters": 1, "schedule_words": 2}
+RUNS = list(FUSED_RUNS) + list(SCHED_RUNS)
 
 
 def _run(pkg, plan, run, xs, ys):
-    if run == "schedule":
+    if run in SCHED_RUNS:
+        plan.set(pkg.OPT_SCHED_TRANSPORT, SCHED_RUNS[run])
         plan.allreduce_schedule(xs, ys)
     else:
         if FUSED_RUNS[run] == 3 and plan.info()["max_depth"] < 3:
@@ -292,7 +300,8 @@ def test_invalid_arguments(pkg):
     ("float32", 32, 65541, 4, 7), ("int32", 7, 1000, 4, 3), ("mat2x2u32", 36, 4099, 16, 5),
     ("float32", 1152, 4099, 3, 2), ("int32", 2, 333, 1, 64), ("float32", 1, 17, 2, 3)])
 @pytest.mark.parametrize("layout", ["aligned", "in_place", "four_byte"])
-def test_schedule_column_slices(pkg, orc, kind, p, m, b, slices, layout):
+@pytest.mark.parametrize("transport", list(TRANSPORTS))
+def test_schedule_column_slices(pkg, orc, kind, p, m, b, slices, layout, transport):
     """Several CTAs per virtual rank, each running the schedule on its own
     column slice of every block, give the same bits."""
     x = host_inputs(kind, 61, p, m)
@@ -303,7 +312,71 @@ def test_schedule_column_slices(pkg, orc, kind, p, m, b, slices, layout):
     ys, keep_y = (xs, None) if layout == "in_place" else empty_like_ranks(xs, pad_front=pad)
     with pkg.Plan(p, m, kind, b) as plan:
         plan.set(pkg.OPT_SCHED_SLICES, slices)
+        plan.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[transport])
         assert plan.info()["sched_slices"] == slices
         plan.allreduce_schedule(xs, ys)
         plan.sync()
     _check_all(ys, want)
+
+
+def test_schedule_transport_choice(pkg):
+    """Flagged words while a rank's buffer is at most 32 KiB (and the word
+    arrays fit 1 GiB), counters above; the option overrides either way."""
+    with pkg.Plan(36, 8192, "int32", 0) as plan:
+        assert plan.info()["sched_transport"] == 2
+        plan.set(pkg.OPT_SCHED_TRANSPORT, 1)
+        assert plan.info()["sched_transport"] == 1
+    with pkg.Plan(36, 8193, "int32", 0) as plan:
+        assert plan.info()["sched_transport"] == 1
+        plan.set(pkg.OPT_SCHED_TRANSPORT, 2)
+        assert plan.info()["sched_transport"] == 2
+    with pkg.Plan(36, 2048, "mat2x2u32", 0) as plan:
+        assert plan.info()["sched_transport"] == 2
+    with pkg.Plan(36, 2049, "mat2x2u32", 0) as plan:
+        assert plan.info()["sched_transport"] == 1
+    from paper_2109_12626_gb300 import DpdrError
+    with pkg.Plan(3, 10, "int32", 0) as plan:
+        with pytest.raises(DpdrError):
+            plan.set(pkg.OPT_SCHED_TRANSPORT, 3)
+
+
+@pytest.mark.parametrize("transport", list(TRANSPORTS))
+def test_schedule_graph_replay(pkg, orc, transport):
+    """A CUDA graph of two schedule calls (two plans, the second reducing the
+    first's result) replayed with new input values in between: the
+    flagged-word transport moves to a new epoch on the device at the end of
+    every call, so a replay never accepts a previous call's words."""
+    kind, p, m = "int32", 30, 777
+    dev = torch.device("cuda:0")
+    xs = [torch.empty(m, dtype=torch.int32, device=dev) for _ in range(p)]
+    ys = [torch.empty(m, dtype=torch.int32, device=dev) for _ in range(p)]
+    zs = [torch.empty(m, dtype=torch.int32, device=dev) for _ in range(p)]
+    with pkg.Plan(p, m, kind, 3) as plan, pkg.Plan(p, m, kind, 2) as plan2:
+        for pl in (plan, plan2):
+            pl.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[transport])
+        first, second = plan.bind(xs, ys), plan2.bind(ys, zs)
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):  # warm-up outside the capture
+            first.allreduce_schedule()
+            second.allreduce_schedule()
+        torch.cuda.current_stream().wait_stream(s)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            first.allreduce_schedule()
+            second.allreduce_schedule()
+        for seed in (31, 32, 33):
+            x = host_inputs(kind, seed, p, m, lo=-1000, hi=1000)
+            for i in range(p):
+                xs[i].copy_(torch.from_numpy(x[i]))
+            for t in ys + zs:
+                t.fill_(-7)
+            g.replay()
+            torch.cuda.synchronize()
+            want = _want(orc, x, kind)
+            _check_all(ys, want)
+            y = np.stack([want.view(np.int32)] * p)
+            _check_all(zs, _want(orc, y, kind))
+        plan.sync()
+        plan2.sync()
