@@ -306,6 +306,9 @@ def model_rounds(p: int, topology: str = "dual") -> int:
     return max(1, 4 * h - (4 if topology == "single" else 7))
 
 
+TRANSPORTS = {"auto": 0, "counters": 1, "words": 2}
+
+
 def fit_cost_model(p: int, m: int, points, topology: str = "dual"):
     """Least-squares fit of T(b) = T0 + (L + 3(b-1)) (alpha + beta m / b)
     (Sec. 1.2's cost model plus a launch constant T0) to (b, seconds)
@@ -374,6 +377,7 @@ def run_sweep(args, w) -> int:
                    "topology": args.topology}
             b0 = -(-m // args.block_size) if args.block_size else 0
             with pkg.Plan(p, m, kind, b0, topology=args.topology) as plan:
+                plan.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[args.transport])
                 bd = plan.bind(xs, ys)
                 t = _timed(lambda: bd.allreduce(), 20, None, graph=True)
                 info = plan.info()
@@ -400,13 +404,14 @@ def run_sweep(args, w) -> int:
     points = []
     for b in bs:
         with pkg.Plan(p, m, kind, b, topology=args.topology) as plan:
+            plan.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[args.transport])
             bd = plan.bind(xs, ys)
             t = _timed(lambda: bd.allreduce_schedule(), 5 if m >= (1 << 20) else 10, None,
                        graph=True)
             plan.sync()
             points.append((b, t))
             print(json.dumps({"sweep": "b", "workload": args.workload, "topology": args.topology,
-                              "p": p, "m": m, "b": b,
+                              "transport": args.transport, "p": p, "m": m, "b": b,
                               "us": round(t * 1e6, 2), "slices": plan.info()["sched_slices"]}),
                   flush=True)
     t0, alpha, beta = fit_cost_model(p, m, points, args.topology)
@@ -414,7 +419,7 @@ def run_sweep(args, w) -> int:
     kappa = alpha / beta if beta > 0 else float("inf")
     rule = pkg.block_count_rule(p, m, kappa) if beta > 0 and alpha > 0 else None
     print(json.dumps({"sweep": "b-fit", "workload": args.workload, "topology": args.topology,
-                      "p": p, "m": m,
+                      "transport": args.transport, "p": p, "m": m,
                       "rounds_L": model_rounds(p, args.topology), "T0_us": round(t0 * 1e6, 3),
                       "alpha_us": round(alpha * 1e6, 4), "beta_ns_per_elem": round(beta * 1e9, 5),
                       "kappa_elems": round(kappa, 1) if beta > 0 else None,
@@ -451,6 +456,8 @@ def main(argv=None) -> int:
     ap.add_argument("--mlist", default=None, help="comma-separated m values for --sweep m")
     ap.add_argument("--host-path", type=int, default=0,
                     help="e2e leg: 0 direct when possible, 1 copy pipeline, 2 direct")
+    ap.add_argument("--transport", choices=tuple(TRANSPORTS), default="auto",
+                    help="schedule kernel: how blocks pass between virtual ranks")
     args = ap.parse_args(argv)
     args.warmup = max(args.warmup, 3)
 
@@ -487,6 +494,7 @@ def main(argv=None) -> int:
     xs = gen_device_inputs(w, dev)
     ys = [torch.empty_like(x) for x in xs]
     plan = pkg.Plan(p, m, kind, b, topology=args.topology)
+    plan.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[args.transport])
     if args.split_depth is not None:
         plan.set(pkg.OPT_SPLIT_DEPTH, args.split_depth)
     if args.mode:

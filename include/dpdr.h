@@ -123,10 +123,16 @@ int dpdr_block_count_rule(int p, int64_t m, double kappa);
  * of m elements of (dtype, op) on the current CUDA device, and allocates the
  * plan's device scratch (rank-pointer tables, handshake counters, the dual
  * roots' exchange slots, an error word, and the word arrays of the
- * schedule kernel's flagged-word transport when it is selected).  b is the number of pipeline
- * blocks (Algorithm 1); b == 0 selects dpdr_block_count_rule(p, m, 0);
- * b is clamped to [1, max(m,1)].  p >= 1, m >= 0.  Returns NULL on error
- * (see dpdr_last_error).  Not thread-safe with respect to one plan. */
+ * schedule kernel's flagged-word transport when it is selected).  b is the
+ * number of pipeline blocks (Algorithm 1), clamped to [1, max(m,1)].
+ * b == 0 selects a block count measured for the schedule kernel on this
+ * GPU: 1 when the flagged-word transport is selected (latency-bound);
+ * otherwise dpdr_block_count_rule(p, m, kappa) with kappa = 46e6 / (p
+ * esize) elements (alpha/beta of the counters transport; the ranks share
+ * device memory, so beta grows with p), raised to at least
+ * 4 p m esize / (L2 bytes) so that the blocks in flight stay in L2.
+ * p >= 1, m >= 0.  Returns NULL on error (see dpdr_last_error).  Not
+ * thread-safe with respect to one plan. */
 dpdr_plan_t dpdr_plan(int p, int64_t m, dpdr_dtype dtype, dpdr_op op, int b);
 
 /* dpdr_plan for either topology (dpdr_plan is DPDR_TOPO_DUAL).  Every entry
@@ -283,7 +289,8 @@ int dpdr_plan_sync(dpdr_plan_t plan, dpdr_stream_t stream);
  *
  * x and y are host arrays of p device pointers, as for dpdr_allreduce; the
  * caller guarantees that no buffers overlap except y[i] == x[i] (this call
- * does not check overlap).  b as for dpdr_plan (0 = block-count rule).
+ * does not check overlap).  b: pipeline blocks, clamped to [1, m];
+ * 0 selects dpdr_block_count_rule(p, m, 0).
  * The call is synchronous: it returns after stream has finished the
  * kernel, with DPDR_ERR_TIMEOUT if one of its bounded waits expired.  The
  * first call on each device looks up the array's device address (with that

@@ -38,6 +38,7 @@ struct Plan {
     size_t esize = 4;
     int device = 0;
     int num_sms = 0;
+    int l2_bytes = 0;
 
     // trees (Sec. 1.1)
     std::vector<int> parent, child0, child1, dual, depth;

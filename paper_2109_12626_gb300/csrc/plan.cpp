@@ -180,6 +180,34 @@ static int clamp_b(int64_t m, int64_t b)
                                                       int64_t(1) << 30)));
 }
 
+// Block count for b == 0 (dpdr_plan, DPDR_OPT_BLOCKS 0): the Sec. 1.2
+// optimum b* = sqrt((4h-6) m / (3 kappa)) with kappa = alpha/beta as
+// measured for the schedule kernel on GB300, raised so that the blocks the
+// p ranks hold at once fit in L2.
+//  * counters transport: alpha is 2.2-2.7 us per round and beta grows with
+//    p (the virtual ranks share HBM), so kappa ~ kKappaBytes / (p esize):
+//    about 40 K elements at p = 288 and 10 K at p = 1152 for int32, the
+//    best b of b sweeps at m = 2^14 .. 2^18.  From m ~ 2^20 the best b is
+//    larger: the partial and final blocks stay in L2 when about four blocks
+//    per rank (input, partial, final, the next block) fit, so
+//    b >= 4 p m esize / L2 (p = 1152, m = 2^22: 14.7 ms at b = 512 against
+//    17.9 ms at b = 128).
+//  * flagged-word transport (m esize <= 32 KiB): latency-bound, b = 1.
+constexpr double kKappaBytes = 46e6;
+
+static int default_blocks(const Plan* P)
+{
+    if (schedule_transport(P) == 2) return 1;
+    const double kappa = std::max(1.0, kKappaBytes / (double(P->p) * double(P->esize)));
+    int64_t b = block_count_rule(P->p, P->m, kappa);
+    if (P->l2_bytes > 0) {
+        const double need = 4.0 * double(P->p) * double(P->m) * double(P->esize) /
+                            double(P->l2_bytes);
+        b = std::max<int64_t>(b, int64_t(std::ceil(need)));
+    }
+    return clamp_b(P->m, b);
+}
+
 static void build_tables(Plan* P)
 {
     const int p = P->p;
@@ -333,7 +361,6 @@ extern "C" dpdr_plan_t dpdr_plan_topo(int p, int64_t m, dpdr_dtype dtype, dpdr_o
     P->dtype = dtype;
     P->op = op;
     P->esize = (dtype == DPDR_MAT2X2_U32 || dtype == DPDR_MAT2X2_F32) ? 16 : 4;
-    P->b = clamp_b(m, b == 0 ? block_count_rule(p, m, 0) : b);
     build_tables(P);
     if (P->max_depth > kMaxDepth) {
         fail(DPDR_ERR_INVALID, "dpdr_plan: p too large");
@@ -343,11 +370,14 @@ extern "C" dpdr_plan_t dpdr_plan_topo(int p, int64_t m, dpdr_dtype dtype, dpdr_o
     cudaError_t e = cudaGetDevice(&P->device);
     if (e == cudaSuccess)
         e = cudaDeviceGetAttribute(&P->num_sms, cudaDevAttrMultiProcessorCount, P->device);
+    if (e == cudaSuccess)
+        e = cudaDeviceGetAttribute(&P->l2_bytes, cudaDevAttrL2CacheSize, P->device);
     if (e != cudaSuccess) {
         cuda_fail(e, "dpdr_plan: device query");
         free_plan(P);
         return nullptr;
     }
+    P->b = b == 0 ? default_blocks(P) : clamp_b(m, b);
     if (allocate(P) != DPDR_OK || schedule_configure(P) != DPDR_OK ||
         (schedule_transport(P) == 2 && schedule_ll_prepare(P) != DPDR_OK) ||
         fused_split_prepare(P, false, P->split_depth) != DPDR_OK) {
@@ -436,7 +466,7 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
         return DPDR_OK;
     case DPDR_OPT_BLOCKS: {
         if (v < 0) return fail(DPDR_ERR_INVALID, "b < 0");
-        const int nb = clamp_b(P->m, v == 0 ? block_count_rule(P->p, P->m, 0) : v);
+        const int nb = v == 0 ? default_blocks(P) : clamp_b(P->m, v);
         Plan tmp;
         tmp.m = P->m;
         tmp.b = nb;

@@ -380,3 +380,20 @@ def test_schedule_graph_replay(pkg, orc, transport):
             _check_all(zs, _want(orc, y, kind))
         plan.sync()
         plan2.sync()
+
+
+def test_default_block_count(pkg):
+    """b == 0: one block with flagged words; otherwise the Sec. 1.2 rule at
+    kappa = 46e6 / (p esize), raised to 4 p m esize / L2 blocks."""
+    import math
+    l2 = torch.cuda.get_device_properties(0).L2_cache_size
+    with pkg.Plan(288, 2500, "int32", 0) as plan:
+        assert plan.info()["sched_transport"] == 2 and plan.query()["b"] == 1
+    for p, m in ((288, 65536), (1152, 16384), (1152, 1 << 22), (36, 1 << 20)):
+        with pkg.Plan(p, m, "int32", 0) as plan:
+            assert plan.info()["sched_transport"] == 1
+            rule = pkg.block_count_rule(p, m, 46e6 / (p * 4))
+            want = max(rule, math.ceil(4 * p * m * 4 / l2))
+            assert plan.query()["b"] == want, (p, m)
+            plan.set(pkg.OPT_BLOCKS, 0)
+            assert plan.query()["b"] == want
