@@ -8,9 +8,10 @@ y_i receives x_0 (.) ... (.) x_{p-1} (one launch of the fused kernel, or of
 the schedule kernel with --kernel schedule).  Inputs are seeded synthetic
 vectors generated on the device before timing (counter-based generator of
 paper_2109_12626_gb300.inputs).  The metric is GB/s = 2 p m sizeof / t (p m
-elements read plus p m written) over K timed steps after W warm-up steps;
-the inputs (and outputs) are larger than the 129 MB L2, so no flush is
-needed between steps.
+elements read plus p m written) over K timed steps after W warm-up steps.
+Inputs larger than twice the L2 (the default workload's 17 GB) need no flush
+between steps; smaller ones get a write of twice the L2 before every step,
+and the time is then the sum of the steps' own CUDA-event intervals.
 
 The JSON line also carries
   e2e           the same metric with pinned host buffers: per step the host
@@ -52,7 +53,8 @@ KERNEL_SOURCES = {"stream": ("fused_stream.cu", "fused_common.cuh"),
                   "tile": ("fused_tile.cu", "fused_common.cuh"),
                   "split": ("fused_split.cu", "fused_common.cuh"),
                   "bulk": ("fused_bulk.cu", "fused_common.cuh"),
-                  "schedule": ("schedule.cu",)}
+                  "schedule": ("schedule.cu", "schedule_common.cuh"),
+                  "schedule_words": ("schedule_ll.cu", "schedule_common.cuh")}
 LAYOUTS = {1: "stream", 2: "tile", 3: "split", 4: "bulk"}
 
 
@@ -514,11 +516,18 @@ def main(argv=None) -> int:
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     bound = plan.bind(xs, ys)
     go = bound.allreduce if args.kernel == "fused" else bound.allreduce_schedule
+    # inputs that L2 could hold: write a buffer of twice L2 before every step
+    # and time the steps by their own events, so each step starts cold
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    flush = (torch.empty(2 * l2 // 4, dtype=torch.int32, device=dev)
+             if p * m * es < 2 * l2 else None)
     barrier(world)
     torch.cuda.synchronize(dev)
     torch.cuda.nvtx.range_push("dpdr_timed")
     start.record(stream)
     for k in range(args.steps):
+        if flush is not None:
+            flush.fill_(k)
         ev[k][0].record(stream)
         go(stream)
         ev[k][1].record(stream)
@@ -528,8 +537,8 @@ def main(argv=None) -> int:
     barrier(world)
     clocks = sampler.stop()
     plan.sync(stream)
-    total_ms = start.elapsed_time(stop)
     launch_ms = [a.elapsed_time(z) for a, z in ev]
+    total_ms = start.elapsed_time(stop) if flush is None else sum(launch_ms)
     t_max = max_over_ranks(total_ms, world, dev)
     ms_per_step = t_max / args.steps
     value = world * algo_bytes / (ms_per_step * 1e-3) / 1e9
@@ -584,7 +593,8 @@ def main(argv=None) -> int:
                "sample": sample}
 
     info = plan.info()
-    layout = LAYOUTS[args.mode or info["auto_mode"]] if args.kernel == "fused" else "schedule"
+    layout = (LAYOUTS[args.mode or info["auto_mode"]] if args.kernel == "fused"
+              else ("schedule", "schedule_words")[info["sched_transport"] - 1])
     launches_per_step = 2 if layout == "split" else 1
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s",
@@ -598,8 +608,10 @@ def main(argv=None) -> int:
                    "fused_mode": args.mode or info["auto_mode"],
                    "split_depth": info["split_depth"] if (args.mode or info["auto_mode"]) == 3 else None,
                    "bytes_per_step": algo_bytes,
-                   "l2": "inputs larger than L2 (%.1f GB), no flush" % (algo_bytes / 2e9)
-                   if algo_bytes / 2 > 129e6 else "working set fits L2: warm-cache number",
+                   "l2": ("inputs larger than twice L2 (%.1f GB), no flush" % (algo_bytes / 2e9)
+                          if flush is None else
+                          "L2 flushed before every step (a 2 x L2 write); time = sum of the "
+                          "steps' own CUDA-event intervals"),
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "roofline": {"bound": "hbm", "kernel": layout, "achieved": round(achieved, 1), "peak": peak,
                      "unit": "GB/s", "frac": round(achieved / peak, 4),

@@ -90,28 +90,44 @@ __device__ __forceinline__ int64_t slice_at(const SchedArgs& a, int64_t s, int64
     return sched::slice_bound<EPV>(s, e, g, a.nslices);
 }
 
-// Thread 0 waits for *ctr >= target within the plan's time bound; the CTA
-// learns the outcome through shared memory.  Returns false on timeout or
-// abort (then the caller returns from the kernel).
-__device__ __forceinline__ bool cta_wait(const SchedArgs& a, const uint32_t* ctr, uint32_t target,
-                         int rank, int j, int step)
+// One counter wait: *ctr >= target; step names the exchange for the error
+// record (0 child_0, 1 child_1, 2 dual, 3 parent).
+struct Wait {
+    const uint32_t* ctr;
+    uint32_t target;
+    int step;
+};
+
+// Thread 0 waits until every one of the n counters (n <= 3, the same on all
+// threads) reaches its target, polling them together within the plan's time
+// bound; the CTA learns the outcome through shared memory.  Returns false on
+// timeout or abort (then the caller returns from the kernel).
+__device__ __forceinline__ bool cta_wait(const SchedArgs& a, const Wait* w, int n, int rank,
+                                         int j)
 {
+    if (n == 0) return true;
     __shared__ int ok;
     if (threadIdx.x == 0) {
         int r = 1;
-        if (ld_acquire(ctr) < target) {
+        unsigned pending = 0;
+        for (int k = 0; k < n; k++)
+            if (ld_acquire(w[k].ctr) < w[k].target) pending |= 1u << k;
+        if (pending) {
             // poll hot first (a partner is usually a few hundred ns away),
             // then back off gently; every poll checks the time bound
             const uint64_t t0 = now_ns();
             unsigned sleep = 0, polls = 0;
             while (true) {
-                if (ld_acquire(ctr) >= target) break;
+                for (int k = 0; k < n; k++)
+                    if (((pending >> k) & 1u) && ld_acquire(w[k].ctr) >= w[k].target)
+                        pending &= ~(1u << k);
+                if (!pending) break;
                 if ((polls & 15) == 15 && ld_relaxed(a.abort_flag)) { r = 0; break; }
                 if (now_ns() - t0 > uint64_t(a.wait_ns)) {
                     if (atomicCAS(a.err, 0u, uint32_t(DPDR_ERR_TIMEOUT)) == 0u) {
                         a.err[1] = uint32_t(rank);
                         a.err[2] = uint32_t(j);
-                        a.err[3] = uint32_t(step);
+                        a.err[3] = uint32_t(w[__ffs(pending) - 1].step);
                     }
                     __threadfence();
                     atomicExch(a.abort_flag, 1u);
@@ -133,21 +149,28 @@ __device__ __forceinline__ bool cta_wait(const SchedArgs& a, const uint32_t* ctr
 }
 
 // Release the CTA's writes to the rank's partner(s): the barrier orders
-// every thread's block writes before thread 0's gpu-scope release store
+// every thread's block writes before thread 0's gpu-scope release stores
 // (release is cumulative over what thread 0 has observed), and the partner's
-// acquire load orders its reads after it.
-__device__ __forceinline__ void publish(const SchedArgs& a, uint32_t* ctr, uint32_t v, int rank)
+// acquire load orders its reads after them.  ctr1 may be null.
+__device__ __forceinline__ void publish(const SchedArgs& a, uint32_t* ctr0, uint32_t v0,
+                                        uint32_t* ctr1, uint32_t v1, int rank)
 {
     __syncthreads();
-    if (threadIdx.x == 0 && rank != a.skip_rank) st_release(ctr, v);
+    if (threadIdx.x == 0 && rank != a.skip_rank) {
+        st_release(ctr0, v0);
+        if (ctr1) st_release(ctr1, v1);
+    }
 }
 
 // dst[k] = lo[k] (.) hi[k] for k in [s, e); rows are virtual bases indexed
 // by global element number.  dst may equal hi.  With lo == nullptr it is a
-// plain copy dst[k] = hi[k].
+// plain copy dst[k] = hi[k].  Each thread owns the same elements in every
+// call over the same range, so a later call may read what an earlier one
+// wrote without a barrier.  Not inlined: its eight 16-byte registers in
+// flight then fit the 64-register budget without spilling the caller's state.
 template <class Op>
-__device__ __forceinline__ void block_op(const SchedArgs& a, char* dst, const char* lo,
-                         const char* hi, int64_t s, int64_t e)
+__device__ __noinline__ void block_op(const SchedArgs& a, char* dst, const char* lo,
+                                         const char* hi, int64_t s, int64_t e)
 {
     constexpr int EPV = Op::kEpv;
     constexpr int ES = Op::kEsize;
@@ -191,6 +214,18 @@ __device__ __forceinline__ void block_op(const SchedArgs& a, char* dst, const ch
     }
 }
 
+// dst = t1 (.) (t0 (.) x) over [s, e) for the children's partial blocks
+// t0, t1 (null when the child does not exist; both null: a copy of x): two
+// passes, the second reading back this thread's own results of the first.
+template <class Op>
+__device__ __forceinline__ void fold_children(const SchedArgs& a, char* dst, const char* t0,
+                                              const char* t1, const char* x, int64_t s,
+                                              int64_t e)
+{
+    block_op<Op>(a, dst, t0, x, s, e);
+    if (t1) block_op<Op>(a, dst, t1, dst, s, e);
+}
+
 __device__ __forceinline__ char* ring_base(const SchedArgs& a, int side, int j,
                                            int64_t s, int epv, int es)
 {
@@ -198,6 +233,12 @@ __device__ __forceinline__ char* ring_base(const SchedArgs& a, int side, int j,
     return slot - (s - s % epv) * es;  // keeps element k congruent mod 16
 }
 
+// Round j of Algorithm 1 at rank i, column slice g.  The waits for the two
+// children's partial blocks do not depend on each other, so thread 0 polls
+// them together, and the folds Y[j] = t1 (.) (t0 (.) x_i) (child_0's partial
+// first, as the steps run) follow without a barrier between them.  The partial goes up before the wait for
+// the parent's final block, so a parent's round j never waits for its own
+// round j-1 to reach the child and come back.
 template <class Op>
 __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j, int g)
 {
@@ -214,61 +255,61 @@ __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j, int 
     const bool inb = j < a.b;
     const int64_t bs = inb ? blk_start(a, j) : 0, be = inb ? blk_start(a, j + 1) : 0;
     const int64_t s = slice_at<EPV>(a, bs, be, g), e = slice_at<EPV>(a, bs, be, g + 1);
-    const int side = (i == a.r0) ? 0 : 1;
-    char* dst = paired_root ? ring_base(a, side, j, bs, Op::kEpv, Op::kEsize) : yi;
 
-    // steps 1 and 2: child_0 then child_1; the send half (final block
-    // j-(d+1)) is read by the child itself from y_i once down[i] covers it
-    bool have = false;
-    for (int k = 0; k < 2; k++) {
-        const int c = k ? c1 : c0;
-        if (c < 0 || !inb) continue;
-        if (!cta_wait(a, up + c, uint32_t(j + 1), i, j, k)) return false;
-        const bool leaf = __ldg(a.child0 + c) < 0;
-        const char* src = leaf
-            ? rank_in(a.x, c)
-            : rank_in(a.y, c);
-        block_op<Op>(a, dst, src, have ? dst : xi, s, e);  // Y[j] = t (.) Y[j]
-        have = true;
-        __syncthreads();
+    // steps 1 and 2: the children's partial blocks (a leaf's is x_c, an inner
+    // node's y_c); the send half (final block j-(d+1)) is read by the child
+    // itself from y_i once down[i] covers it
+    const char* t[2] = {nullptr, nullptr};
+    if (inb) {
+        Wait w[2];
+        int n = 0;
+        for (int k = 0; k < 2; k++) {
+            const int c = k ? c1 : c0;
+            if (c < 0) continue;
+            t[k] = __ldg(a.child0 + c) < 0 ? rank_in(a.x, c) : rank_in(a.y, c);
+            w[n++] = Wait{up + c, uint32_t(j + 1), k};
+        }
+        if (!cta_wait(a, w, n, i, j)) return false;
     }
 
     if (paired_root) {  // step 3 at a root: exchange partials with the dual
         if (!inb) return true;
-        if (!have) {
-            block_op<Op>(a, dst, nullptr, xi, s, e);
-            __syncthreads();
-        }
-        publish(a, up + i, uint32_t(j + 1), i);
+        const int side = (i == a.r0) ? 0 : 1;
+        char* slot = ring_base(a, side, j, bs, Op::kEpv, Op::kEsize);
+        fold_children<Op>(a, slot, t[0], t[1], xi, s, e);
+        publish(a, up + i, uint32_t(j + 1), nullptr, 0, i);
         const int du = (i == a.r0) ? a.r1 : a.r0;
-        if (!cta_wait(a, up + du, uint32_t(j + 1), i, j, 2)) return false;
+        const Wait wd{up + du, uint32_t(j + 1), 2};
+        if (!cta_wait(a, &wd, 1, i, j)) return false;
         const char* other = ring_base(a, 1 - side, j, bs, Op::kEpv, Op::kEsize);
         if (i == a.r0)
-            block_op<Op>(a, yi, dst, other, s, e);  // lower root: Y[j] (.) t
+            block_op<Op>(a, yi, slot, other, s, e);  // lower root: Y[j] (.) t
         else
-            block_op<Op>(a, yi, other, dst, s, e);  // higher root: t (.) Y[j]
-        publish(a, down + i, uint32_t(j + 1), i);
+            block_op<Op>(a, yi, other, slot, s, e);  // higher root: t (.) Y[j]
+        publish(a, down + i, uint32_t(j + 1), nullptr, 0, i);
         return true;
     }
     if (root) {  // the root of a single tree (or p == 1): its block is final
         if (!inb) return true;
-        if (!have && xi != yi) {
-            block_op<Op>(a, yi, nullptr, xi, s, e);
-            __syncthreads();
-        }
-        publish(a, down + i, uint32_t(j + 1), i);
+        if (t[0] || xi != yi) fold_children<Op>(a, yi, t[0], t[1], xi, s, e);
+        publish(a, down + i, uint32_t(j + 1), nullptr, 0, i);
         return true;
     }
-    // step 3 elsewhere: partial Y[j] up (in y_i, or x_i for a leaf), final
-    // Y[j-d] down from the parent
-    if (inb) publish(a, up + i, uint32_t(j + 1), i);
+    // step 3 elsewhere: partial Y[j] up (in y_i, or x_i itself for a leaf),
+    // final Y[j-d] down from the parent
+    if (inb) {
+        if (t[0]) fold_children<Op>(a, yi, t[0], t[1], xi, s, e);
+        publish(a, up + i, uint32_t(j + 1), nullptr, 0, i);
+    }
     const int kf = j - d;
     if (kf >= 0 && kf < a.b) {
-        if (!cta_wait(a, down + par, uint32_t(kf + 1), i, j, 3)) return false;
+        const Wait wp{down + par, uint32_t(kf + 1), 3};
+        if (!cta_wait(a, &wp, 1, i, j)) return false;
         const char* yp = rank_in(a.y, par);
         const int64_t ks = blk_start(a, kf), ke = blk_start(a, kf + 1);
-        block_op<Op>(a, yi, nullptr, yp, slice_at<EPV>(a, ks, ke, g), slice_at<EPV>(a, ks, ke, g + 1));
-        publish(a, down + i, uint32_t(kf + 1), i);
+        block_op<Op>(a, yi, nullptr, yp, slice_at<EPV>(a, ks, ke, g),
+                     slice_at<EPV>(a, ks, ke, g + 1));
+        publish(a, down + i, uint32_t(kf + 1), nullptr, 0, i);
     }
     return true;
 }
