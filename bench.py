@@ -53,9 +53,10 @@ KERNEL_SOURCES = {"stream": ("fused_stream.cu", "fused_common.cuh"),
                   "tile": ("fused_tile.cu", "fused_common.cuh"),
                   "split": ("fused_split.cu", "fused_common.cuh"),
                   "bulk": ("fused_bulk.cu", "fused_common.cuh"),
+                  "tree": ("fused_tree.cu", "fused_common.cuh"),
                   "schedule": ("schedule.cu", "schedule_common.cuh"),
                   "schedule_words": ("schedule_ll.cu", "schedule_common.cuh")}
-LAYOUTS = {1: "stream", 2: "tile", 3: "split", 4: "bulk"}
+LAYOUTS = {1: "stream", 2: "tile", 3: "split", 4: "bulk", 5: "tree"}
 
 
 # ------------------------------------------------------------ workload
@@ -441,7 +442,8 @@ def main(argv=None) -> int:
     ap.add_argument("--m", type=int, default=None, help="override m (sweeps)")
     ap.add_argument("--kernel", choices=("fused", "schedule"), default="fused")
     ap.add_argument("--b", type=int, default=None, help="pipeline blocks (schedule)")
-    ap.add_argument("--mode", type=int, default=0, help="fused layout: 0 auto, 1, 2, 3")
+    ap.add_argument("--mode", type=int, default=0,
+                    help="fused layout: 0 auto, 1 stream, 2 tile, 3 split, 4 bulk, 5 tree")
     ap.add_argument("--split-depth", type=int, default=None, help="split layout cut depth")
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-e2e", action="store_true")

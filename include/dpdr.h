@@ -148,11 +148,12 @@ int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
 
 /* Plan options (key, value):
  *   DPDR_OPT_FUSED_MODE       0 auto, 1 column-streaming, 2 shared-memory
- *                             tile, 3 subtree split, 4 bulk-copy pipeline
- *                             (the four layouts of dpdr_allreduce; 3 needs
- *                             p >= 2 and keeps m * esize bytes of scratch
- *                             per subtree; 4 needs 16-byte aligned buffers
- *                             and otherwise runs as 1)
+ *                             tile, 3 subtree split, 4 bulk-copy pipeline,
+ *                             5 hierarchical tile (the five layouts of
+ *                             dpdr_allreduce; 3 needs p >= 2 and keeps
+ *                             m * esize bytes of scratch per subtree; 4 and
+ *                             5 need 16-byte aligned buffers and otherwise
+ *                             run as 1)
  *   DPDR_OPT_WAIT_LIMIT_NS    bound of every wait of the schedule kernel,
  *                             nanoseconds (default 4e9)
  *   DPDR_OPT_SKIP_RANK        fault injection for tests: this rank of the

@@ -23,7 +23,7 @@ INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 SOURCES = ["plan.cpp", "api.cpp", "fused.cu", "fused_stream.cu", "fused_tile.cu",
            "fused_split.cu", "fused_bulk.cu", "schedule.cu",
-           "schedule_ll.cu"]
+           "schedule_ll.cu", "fused_tree.cu"]
 
 
 def nvcc() -> str:

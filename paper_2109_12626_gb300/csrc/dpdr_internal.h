@@ -49,7 +49,7 @@ struct Plan {
     std::vector<int> level_off;                // nlevels + 1
 
     // options
-    int fused_mode = 0;        // 0 auto, 1 stream, 2 tile, 3 split, 4 bulk
+    int fused_mode = 0;        // 0 auto, 1 stream, 2 tile, 3 split, 4 bulk, 5 tree
     int64_t wait_ns = 4000000000LL;
     int skip_rank = -1;
     int sched_threads = 128;
@@ -90,7 +90,7 @@ struct Plan {
 
     // dynamic shared memory already granted to the fused kernels of this
     // plan's element type (stream, tile), so launches skip the attribute call
-    int smem_attr[4] = {48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024};
+    int smem_attr[5] = {48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024};
 
     // split layout of the fused kernel (fused.cu): subtrees at depth split_s
     bool split_ready = false;
@@ -101,6 +101,16 @@ struct Plan {
     int2* d_items = nullptr;
     char* d_part = nullptr;
     int64_t part_stride = 0;
+
+    // hierarchical tile layout of the fused kernel (fused_tree.cu): entries
+    // (subtrees at depth tree_s, then nodes above the cut) and level table
+    bool tree_ready = false;
+    int tree_s = 0, tree_nseg = 0, tree_nlev = 0, tree_slots = 0, tree_r0 = -1, tree_r1 = 0;
+    char* d_tree = nullptr;          // own allocation
+    size_t d_tree_bytes = 0;
+    int2* d_tree_seg = nullptr;
+    int4* d_tree_lev = nullptr;
+    int* d_tree_levoff = nullptr;
 
     // host-buffer pipeline of dpdr_allreduce_host (api.cpp), made on first use:
     // column chunks copied in on one stream, reduced on the caller's stream,
@@ -145,6 +155,8 @@ int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t m
                       cudaStream_t s, int force_mode);  // fused.cu (0: plan's choice)
 int fused_auto_mode(const Plan* P);             // fused.cu
 int fused_split_prepare(Plan* P, bool force, int depth);  // fused.cu
+int fused_tree_prepare(Plan* P);                // fused_tree.cu
+bool fused_tree_wanted(const Plan* P);          // fused.cu
 int schedule_launch(Plan* P, cudaStream_t s);   // schedule.cu
 int schedule_configure(Plan* P);                // schedule.cu
 int schedule_transport(const Plan* P);          // schedule_ll.cu: 1 counters, 2 words

@@ -12,9 +12,15 @@ using fused::tile_lg_wu;
 // Threads the streaming layouts want in flight to cover HBM latency.
 static int64_t stream_target(const Plan* P) { return int64_t(P->num_sms) * 1024; }
 
-// Layout choice, from layout sweeps measured on GB300:
-//  * deep trees (p >= 128) whose p input rows total at most kTileMaxBytes:
-//    the shared-memory tile, the layout with the lowest fixed cost (p = 288,
+// Layout choice, from layout sweeps measured on GB300 (int32, p = 128 ...
+// 4096, m = 2^10 ... 2^20, warm and cold L2):
+//  * deep trees (p >= 128) with few columns -- at most 2048 16-byte column
+//    units, 4096 from p = 512 -- but more than 20 MB of inputs once
+//    p >= 1024: the hierarchical tile, one kernel with a walk of about
+//    p / 64 ranks per thread (p = 1152, m = 2^13, cold: 21.9 us against
+//    36.4 us for the tile and 38.5 us for the split layout);
+//  * deep trees whose p input rows total at most kTileMaxBytes: the
+//    shared-memory tile, the layout with the lowest fixed cost (p = 288,
 //    m = 2^15 int32: 22.6 us against the split layout's 27.3 us; at 75.5 MB,
 //    twice that, the split layout wins at p = 288, 576 and 1152);
 //  * deep trees (p >= kSplitMinRanks) above that: the split layout, whose
@@ -27,6 +33,16 @@ static int64_t stream_target(const Plan* P) { return int64_t(P->num_sms) * 1024;
 constexpr int64_t kTileMaxBytes = int64_t(40) << 20;
 constexpr int kSplitMinRanks = 128;
 constexpr int64_t kSplitWork = int64_t(1) << 17;
+constexpr int64_t kTreeMinBytesLargeP = int64_t(20) << 20;
+
+static bool tree_preferred(const Plan* P)
+{
+    if (P->p < 128) return false;
+    const int64_t units = P->m * int64_t(P->esize) / 16;
+    const int64_t bytes = int64_t(P->p) * P->m * P->esize;
+    if (units > (P->p >= 512 ? 4096 : 2048)) return false;
+    return P->p < 1024 || bytes > kTreeMinBytesLargeP;
+}
 
 static bool tile_preferred(const Plan* P)
 {
@@ -37,6 +53,7 @@ static bool tile_preferred(const Plan* P)
 int fused_auto_mode(const Plan* P)
 {
     const int64_t units = P->m * int64_t(P->esize) / 16;
+    if (P->tree_ready && tree_preferred(P)) return 5;
     if (tile_preferred(P)) return 2;
     if (P->p >= kSplitMinRanks && units >= 4096 && P->split_ready) return 3;
     if (units >= stream_target(P) / 4) return 1;
@@ -44,12 +61,16 @@ int fused_auto_mode(const Plan* P)
     return P->split_ready ? 3 : 1;
 }
 
+// Whether the automatic choice can be the hierarchical tile (then the plan
+// prepares its tables up front).
+bool fused_tree_wanted(const Plan* P) { return tree_preferred(P); }
+
 // Whether the automatic choice can be the split layout (then the plan
 // prepares it up front).
 static bool split_wanted(const Plan* P)
 {
     const int64_t units = P->m * int64_t(P->esize) / 16;
-    return P->p >= kSplitMinRanks && units >= 4096 && !tile_preferred(P);
+    return P->p >= kSplitMinRanks && units >= 4096 && !tile_preferred(P) && !tree_preferred(P);
 }
 
 // Split layout: cut depth s, subtree table, top-of-tree item list, rank
@@ -140,7 +161,8 @@ int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t m
     const int lg = tile_lg_wu(P);
     if (mode == 2 && lg < 0) return fail(DPDR_ERR_INVALID, "tile mode: p too large");
     if (mode == 3 && !P->split_ready) return fail(DPDR_ERR_INVALID, "split mode: p < 2");
-    if (mode < 1 || mode > 4) return fail(DPDR_ERR_INVALID, "unknown fused mode");
+    if (mode == 5 && !P->tree_ready) return fail(DPDR_ERR_INVALID, "tree mode not prepared");
+    if (mode < 1 || mode > 5) return fail(DPDR_ERR_INVALID, "unknown fused mode");
 
     FusedArgs a;
     a.x = dx;
@@ -169,12 +191,23 @@ int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t m
     a.bulk_bar_off = 0;
     a.err = P->d_err;
     a.wait_ns = P->wait_ns;
-    if (mode == 4 && !vec) mode = 1;  // bulk copies need 16-byte aligned rows
+    a.tree_seg = P->d_tree_seg;
+    a.tree_lev = P->d_tree_lev;
+    a.tree_levoff = P->d_tree_levoff;
+    a.tree_nseg = P->tree_nseg;
+    a.tree_nlev = P->tree_nlev;
+    a.tree_r0 = P->tree_r0;
+    a.tree_r1 = P->tree_r1;
+    a.tree_s = P->tree_s;
+    a.tree_slots = P->tree_slots;
+    a.tree_tiles = (a.nvec + fused::kTreeUnits - 1) / fused::kTreeUnits;
+    if ((mode == 4 || mode == 5) && !vec) mode = 1;  // 16-byte rows only: stream instead
 
     switch (mode) {
     case 1: return fused::launch_stream(P, a, s);
     case 2: return fused::launch_tile(P, a, s);
     case 3: return fused::launch_split(P, a, s);
+    case 5: return fused::launch_tree(P, a, s);
     default: return fused::launch_bulk(P, a, s);
     }
 }

@@ -11,7 +11,8 @@
 // (Algorithm 1) do not change the result, so the kernel tiles by columns.
 // Layouts (one file each): column streaming (fused_stream.cu),
 // shared-memory tile (fused_tile.cu), subtree split (fused_split.cu),
-// bulk-copy pipeline (fused_bulk.cu); fused.cu chooses and launches.
+// bulk-copy pipeline (fused_bulk.cu), hierarchical tile (fused_tree.cu);
+// fused.cu chooses and launches.
 #pragma once
 
 #include <algorithm>
@@ -30,6 +31,8 @@ constexpr int kBulkConsumers = 256;                   // 8 warps
 constexpr int kBulkThreads = kBulkConsumers + 32;     // + producer warp
 constexpr int kBulkTile = kBulkConsumers * 16;        // bytes per rank row piece
 constexpr int kBulkStages = 16;
+constexpr int kTreeThreads = 512;                     // hierarchical tile: threads,
+constexpr int kTreeUnits = 8;                         // and 16-byte column units per CTA
 
 struct FusedArgs {
     const char* const* x;   // [p] rank inputs
@@ -58,6 +61,12 @@ struct FusedArgs {
     int bulk_bar_off;       // byte offset of the mbarriers in shared memory
     uint32_t* err;          // plan error record (an expired pipeline wait)
     int64_t wait_ns;
+    // hierarchical tile layout
+    const int2* tree_seg;   // [tree_nseg] subtree intervals, then nodes above the cut
+    const int4* tree_lev;   // levels above the cut: (node, child_0, child_1) entries
+    const int* tree_levoff; // [tree_nlev + 1]
+    int tree_nseg, tree_nlev, tree_r0, tree_r1, tree_s, tree_slots;
+    int64_t tree_tiles;     // CTAs of kTreeUnits vector units
 };
 
 template <class Op>
@@ -176,6 +185,7 @@ int launch_stream(Plan* P, FusedArgs a, cudaStream_t s);
 int launch_tile(Plan* P, FusedArgs a, cudaStream_t s);
 int launch_split(Plan* P, FusedArgs a, cudaStream_t s);
 int launch_bulk(Plan* P, FusedArgs a, cudaStream_t s);
+int launch_tree(Plan* P, FusedArgs a, cudaStream_t s);
 int tile_lg_wu(const Plan* P);
 
 template <template <class> class L>

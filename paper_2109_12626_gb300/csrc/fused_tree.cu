@@ -1,0 +1,217 @@
+// fused_tree.cu -- hierarchical tile layout of the fused kernel: one CTA per
+// tile of kTreeUnits column units runs the whole fold of its columns.
+//
+//  1. The tree is cut at depth s (Sec. 1.1's trees are complete, so a
+//     depth-s node roots a contiguous post-order interval of ranks).  Each
+//     thread walks one depth-s subtree for one column with the running
+//     post-order fold (loads kStreamAhead ranks ahead) and leaves the
+//     subtree's value in shared memory; the inputs of the nodes above the
+//     cut are loaded there too.
+//  2. The nodes above the cut are evaluated level by level, deepest first,
+//     v(i) = v(child_1) (.) (v(child_0) (.) x_i), all nodes of a level in
+//     parallel; then y = v(r0) (.) v(r1) (or v(root) for one tree).
+//  3. All threads store y to the p outputs.
+//
+// One kernel, no scratch rows in device memory, and every thread has a walk
+// of about p / 2^(s+1) ranks: the layout for large p at mid m, where the
+// column-streaming walk over all p ranks is too long and the subtree-split
+// layout pays for a second kernel and a top fold per store group.  A CTA
+// reads all p rows of its columns before it writes any (barrier between
+// phases 1 and 3), and no other CTA touches those columns, so in-place use
+// is safe.  16-byte units only: buffers that are not all 16-byte aligned go
+// to the streaming layout; a ragged tail of single elements gets one extra
+// CTA that streams them.
+#include <algorithm>
+#include <vector>
+
+#include "fused_common.cuh"
+
+namespace dpdr {
+namespace fused {
+namespace {
+
+// Walk of the subtree [lo, hi] (post-order interval, hi its root) at depth
+// s for unit u: the running fold of fold_step with depths taken relative to
+// s, so the slots hold depths s .. max depth.
+template <class U>
+__device__ __forceinline__ typename U::T walk_subtree(const FusedArgs& a, int lo, int hi,
+                                                      int64_t u, typename U::T* slot,
+                                                      int stride, int s)
+{
+    using T = typename U::T;
+    const unsigned shift = unsigned(s) << 3;  // tape depth field starts at bit 3
+    T acc{};  // set by rank lo, a leaf
+    for (int i0 = lo; i0 <= hi; i0 += kStreamAhead) {
+        T cur[kStreamAhead];
+#pragma unroll
+        for (int k = 0; k < kStreamAhead; k++)
+            if (i0 + k <= hi) cur[k] = U::ld(rank_ptr(a.x, i0 + k), u);
+#pragma unroll
+        for (int k = 0; k < kStreamAhead; k++)
+            if (i0 + k <= hi)
+                fold_step<U>(unsigned(__ldg(a.tape + i0 + k)) - shift, cur[k], acc, slot, stride);
+    }
+    return acc;
+}
+
+template <class Op>
+__global__ void __launch_bounds__(kTreeThreads, 2)
+fused_tree_kernel(FusedArgs a)
+{
+    using V = VecUnit<Op>;
+    constexpr int W = kTreeUnits;
+    extern __shared__ uint4 smem[];
+    const int tid = threadIdx.x;
+    if (blockIdx.x >= a.tree_tiles) {  // ragged tail: fewer than 16 bytes per rank
+        if (tid < a.nscalar)
+            stream_column<OneUnit<Op>>(a, a.scalar_base + tid, one_slots<Op>(smem, tid),
+                                       one_slot_stride<Op>(32));
+        return;
+    }
+    const int64_t u0 = int64_t(blockIdx.x) * W;
+    const int wu = int(lmin(W, a.nvec - u0));
+    uint4* part = smem + a.tree_slots * kTreeThreads;  // [nseg][W] node values
+    uint4* yrow = part + a.tree_nseg * W;              // [W] the result
+
+    // 1. subtree walks and the inputs above the cut
+    const int npairs = a.tree_nseg * W;
+    for (int idx = tid; idx < npairs; idx += kTreeThreads) {
+        const int g = idx / W, c = idx % W;
+        if (c >= wu) continue;
+        const int2 sg = __ldg(a.tree_seg + g);
+        const int64_t u = u0 + c;
+        part[idx] = sg.x == sg.y ? V::ld(rank_ptr(a.x, sg.x), u)
+                                 : walk_subtree<V>(a, sg.x, sg.y, u, smem + tid, kTreeThreads,
+                                                   a.tree_s);
+    }
+    __syncthreads();
+    // 2. the nodes above the cut, deepest level first
+    for (int l = 0; l < a.tree_nlev; l++) {
+        const int beg = __ldg(a.tree_levoff + l), end = __ldg(a.tree_levoff + l + 1);
+        const int cnt = (end - beg) * W;
+        for (int idx = tid; idx < cnt; idx += kTreeThreads) {
+            const int k = idx / W, c = idx % W;
+            if (c >= wu) continue;
+            const int4 e = __ldg(a.tree_lev + beg + k);  // node, child_0, child_1
+            uint4 v = part[e.x * W + c];
+            if (e.y >= 0) v = V::op(part[e.y * W + c], v);
+            if (e.z >= 0) v = V::op(part[e.z * W + c], v);
+            part[e.x * W + c] = v;
+        }
+        __syncthreads();
+    }
+    if (tid < wu) {
+        const uint4 v1 = part[a.tree_r1 * W + tid];
+        yrow[tid] = a.dual ? V::op(part[a.tree_r0 * W + tid], v1) : v1;
+    }
+    __syncthreads();
+    // 3. the result to every output
+    const int nst = a.p * W;
+#pragma unroll 4
+    for (int idx = tid; idx < nst; idx += kTreeThreads) {
+        const int i = idx / W, c = idx % W;
+        if (c < wu) V::st(rank_ptr_w(a.y, i), u0 + c, yrow[c]);
+    }
+}
+
+size_t tree_smem(const Plan* P)
+{
+    const size_t walk = size_t(P->tree_slots) * kTreeThreads + size_t(P->tree_nseg) * kTreeUnits +
+                        kTreeUnits;
+    const size_t tail = size_t(P->max_depth + 2) * 32;  // the tail CTA's slots
+    return std::max(walk, tail) * sizeof(uint4);
+}
+
+template <class Op>
+struct Tree {
+    static int run(Plan* P, FusedArgs a, cudaStream_t s)
+    {
+        const size_t smem = tree_smem(P);
+        const int64_t blocks = a.tree_tiles + (a.nscalar ? 1 : 0);
+        if (blocks > 0x7fffffff) return fail(DPDR_ERR_INVALID, "m too large");
+        if (int(smem) > P->smem_attr[4]) {
+            cudaError_t e = cudaFuncSetAttribute(fused_tree_kernel<Op>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 int(smem));
+            if (e != cudaSuccess) return cuda_fail(e, "fused tree attribute");
+            P->smem_attr[4] = int(smem);
+        }
+        fused_tree_kernel<Op><<<unsigned(blocks), kTreeThreads, smem, s>>>(a);
+        return launched();
+    }
+};
+
+}  // namespace
+
+int launch_tree(Plan* P, FusedArgs a, cudaStream_t s) { return dispatch<Tree>(P, a, s); }
+
+}  // namespace fused
+
+// Tables of the hierarchical tile layout: the cut depth s (about
+// kTreeThreads / kTreeUnits subtrees, one walk per thread), the entries --
+// first the depth-s nodes with their subtree intervals, then the nodes above
+// the cut (lo = hi = the node) -- and, per level above the cut, deepest
+// first, (node, child_0, child_1) as entry indices.
+int fused_tree_prepare(Plan* P)
+{
+    if (P->tree_ready) return DPDR_OK;
+    const int p = P->p;
+    const int trees = P->r0 >= 0 ? 2 : 1;
+    int s = 0;
+    while (trees << s < fused::kTreeThreads / fused::kTreeUnits) s++;
+    s = std::min(s, P->max_depth);
+    std::vector<int> idx(p, -1);
+    std::vector<int2> seg;
+    for (int i = 0; i < p; i++) {
+        if (P->depth[i] != s) continue;
+        int lo = i;  // leftmost leaf of the subtree
+        while (P->child0[lo] >= 0) lo = P->child1[lo] >= 0 ? P->child1[lo] : P->child0[lo];
+        idx[i] = int(seg.size());
+        seg.push_back(make_int2(lo, i));
+    }
+    for (int i = 0; i < p; i++) {
+        if (P->depth[i] >= s) continue;
+        idx[i] = int(seg.size());
+        seg.push_back(make_int2(i, i));
+    }
+    std::vector<int4> lev;
+    std::vector<int> off(1, 0);
+    for (int d = s - 1; d >= 0; d--) {
+        for (int i = 0; i < p; i++) {
+            if (P->depth[i] != d) continue;
+            const int c0 = P->child0[i], c1 = P->child1[i];
+            lev.push_back(make_int4(idx[i], c0 >= 0 ? idx[c0] : -1, c1 >= 0 ? idx[c1] : -1, 0));
+        }
+        off.push_back(int(lev.size()));
+    }
+    const size_t o_lev = (sizeof(int2) * seg.size() + 255) / 256 * 256;
+    const size_t o_off = o_lev + (sizeof(int4) * std::max<size_t>(lev.size(), 1) + 255) / 256 * 256;
+    const size_t bytes = o_off + sizeof(int) * off.size();
+    char* d = nullptr;
+    cudaError_t e = cudaMalloc(&d, bytes);
+    if (e != cudaSuccess) return cuda_fail(e, "tree layout: cudaMalloc");
+    e = cudaMemcpy(d, seg.data(), sizeof(int2) * seg.size(), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess && !lev.empty())
+        e = cudaMemcpy(d + o_lev, lev.data(), sizeof(int4) * lev.size(), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess)
+        e = cudaMemcpy(d + o_off, off.data(), sizeof(int) * off.size(), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) {
+        cudaFree(d);
+        return cuda_fail(e, "tree layout: upload");
+    }
+    P->d_tree = d;
+    P->d_tree_bytes = bytes;
+    P->d_tree_seg = reinterpret_cast<int2*>(d);
+    P->d_tree_lev = reinterpret_cast<int4*>(d + o_lev);
+    P->d_tree_levoff = reinterpret_cast<int*>(d + o_off);
+    P->tree_s = s;
+    P->tree_nseg = int(seg.size());
+    P->tree_nlev = int(off.size()) - 1;
+    P->tree_slots = P->max_depth - s + 1;
+    P->tree_r0 = P->r0 >= 0 ? idx[P->r0] : -1;
+    P->tree_r1 = idx[P->r1];
+    P->tree_ready = true;
+    return DPDR_OK;
+}
+
+}  // namespace dpdr

@@ -250,6 +250,7 @@ static void free_plan(Plan* P)
     if (P->pipe_out) cudaStreamDestroy(P->pipe_out);
     if (P->d_pipe) cudaFree(P->d_pipe);
     if (P->d_split) cudaFree(P->d_split);
+    if (P->d_tree) cudaFree(P->d_tree);
     if (P->d_sched) cudaFree(P->d_sched);
     if (P->d_ll) cudaFree(P->d_ll);
     if (P->h_ptrs) cudaFreeHost(P->h_ptrs);
@@ -380,6 +381,7 @@ extern "C" dpdr_plan_t dpdr_plan_topo(int p, int64_t m, dpdr_dtype dtype, dpdr_o
     P->b = b == 0 ? default_blocks(P) : clamp_b(m, b);
     if (allocate(P) != DPDR_OK || schedule_configure(P) != DPDR_OK ||
         (schedule_transport(P) == 2 && schedule_ll_prepare(P) != DPDR_OK) ||
+        (fused_tree_wanted(P) && fused_tree_prepare(P) != DPDR_OK) ||
         fused_split_prepare(P, false, P->split_depth) != DPDR_OK) {
         free_plan(P);
         return nullptr;
@@ -409,11 +411,15 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
     if (!P) return fail(DPDR_ERR_INVALID, "dpdr_plan_set: NULL plan");
     switch (key) {
     case DPDR_OPT_FUSED_MODE:
-        if (v < 0 || v > 4) return fail(DPDR_ERR_INVALID, "fused mode: 0 to 4");
+        if (v < 0 || v > 5) return fail(DPDR_ERR_INVALID, "fused mode: 0 to 5");
         if (v == 3) {
             int rc = fused_split_prepare(P, true, P->split_depth);
             if (rc) return rc;
             if (!P->split_ready) return fail(DPDR_ERR_INVALID, "split mode needs p >= 2");
+        }
+        if (v == 5) {
+            int rc = fused_tree_prepare(P);
+            if (rc) return rc;
         }
         P->fused_mode = int(v);
         return DPDR_OK;
@@ -489,7 +495,7 @@ extern "C" int dpdr_plan_info(dpdr_plan_t h, int64_t* info, int n)
     const int64_t v[] = {P->p, P->m, P->b, P->max_depth, fused_auto_mode(P),
                          P->sched_ctas, P->sched_ranks_per_cta,
                          int64_t(P->dmem_bytes + P->d_split_bytes + P->d_sched_bytes +
-                                 P->d_ll_bytes),
+                                 P->d_ll_bytes + P->d_tree_bytes),
                          P->last_vector_path, P->split_s, P->split_nseg, P->split_group,
                          P->sched_slices_used, P->topo, P->last_host_path,
                          schedule_transport(P)};

@@ -65,7 +65,7 @@ def _check_all(ys, want, guards=None):
 
 
 @pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
-@pytest.mark.parametrize("mode", [1, 2, 3, 4], ids=["stream", "tile", "split", "bulk"])
+@pytest.mark.parametrize("mode", [1, 2, 3, 4, 5], ids=["stream", "tile", "split", "bulk", "tree"])
 def test_fused_matches_oracle(pkg, orc, case, mode):
     _, kind, seed, p, m, kw, _ = case
     dev = torch.device("cuda:0")
@@ -108,7 +108,8 @@ def test_schedule_matches_oracle(pkg, orc, case, transport):
         assert np.array_equal(bits(xs[i]), expect_bits(x[i]))
 
 
-FUSED_RUNS = {"fused_stream": 1, "fused_tile": 2, "fused_split": 3, "fused_bulk": 4}
+FUSED_RUNS = {"fused_stream": 1, "fused_tile": 2, "fused_split": 3, "fused_bulk": 4,
+              "fused_tree": 5}
 SCHED_RUNS = {"schedule_counters": 1, "schedule_words": 2}
 RUNS = list(FUSED_RUNS) + list(SCHED_RUNS)
 
@@ -291,7 +292,7 @@ def test_invalid_arguments(pkg):
         plan.allreduce(xs, ys)
         plan.sync()
         with pytest.raises(DpdrError):
-            plan.set(N.OPT_FUSED_MODE, 5)
+            plan.set(N.OPT_FUSED_MODE, 6)
         with pytest.raises(DpdrError):
             plan.set(999, 1)
 
