@@ -18,9 +18,9 @@
 // layout pays for a second kernel and a top fold per store group.  A CTA
 // reads all p rows of its columns before it writes any (barrier between
 // phases 1 and 3), and no other CTA touches those columns, so in-place use
-// is safe.  16-byte units only: buffers that are not all 16-byte aligned go
-// to the streaming layout; a ragged tail of single elements gets one extra
-// CTA that streams them.
+// is safe.  Buffers that are not all 16-byte aligned go to the streaming
+// layout; a ragged tail of single elements (fewer than 16 bytes per rank)
+// gets one extra CTA that runs the same three phases on them.
 #include <algorithm>
 #include <vector>
 
@@ -54,24 +54,18 @@ __device__ __forceinline__ typename U::T walk_subtree(const FusedArgs& a, int lo
     return acc;
 }
 
-template <class Op>
-__global__ void __launch_bounds__(kTreeThreads, 2)
-fused_tree_kernel(FusedArgs a)
+// The three phases for wu <= kTreeUnits units starting at u0 (16-byte units
+// with VecUnit, single elements with OneUnit); slot/stride are this
+// thread's walk slots.
+template <class U>
+__device__ __forceinline__ void tree_body(const FusedArgs& a, int64_t u0, int wu, uint4* smem,
+                                          typename U::T* slot, int stride)
 {
-    using V = VecUnit<Op>;
+    using T = typename U::T;
     constexpr int W = kTreeUnits;
-    extern __shared__ uint4 smem[];
     const int tid = threadIdx.x;
-    if (blockIdx.x >= a.tree_tiles) {  // ragged tail: fewer than 16 bytes per rank
-        if (tid < a.nscalar)
-            stream_column<OneUnit<Op>>(a, a.scalar_base + tid, one_slots<Op>(smem, tid),
-                                       one_slot_stride<Op>(32));
-        return;
-    }
-    const int64_t u0 = int64_t(blockIdx.x) * W;
-    const int wu = int(lmin(W, a.nvec - u0));
-    uint4* part = smem + a.tree_slots * kTreeThreads;  // [nseg][W] node values
-    uint4* yrow = part + a.tree_nseg * W;              // [W] the result
+    T* part = reinterpret_cast<T*>(smem + a.tree_slots * kTreeThreads);  // [nseg][W]
+    T* yrow = part + a.tree_nseg * W;                                      // [W]
 
     // 1. subtree walks and the inputs above the cut
     const int npairs = a.tree_nseg * W;
@@ -80,9 +74,8 @@ fused_tree_kernel(FusedArgs a)
         if (c >= wu) continue;
         const int2 sg = __ldg(a.tree_seg + g);
         const int64_t u = u0 + c;
-        part[idx] = sg.x == sg.y ? V::ld(rank_ptr(a.x, sg.x), u)
-                                 : walk_subtree<V>(a, sg.x, sg.y, u, smem + tid, kTreeThreads,
-                                                   a.tree_s);
+        part[idx] = sg.x == sg.y ? U::ld(rank_ptr(a.x, sg.x), u)
+                                 : walk_subtree<U>(a, sg.x, sg.y, u, slot, stride, a.tree_s);
     }
     __syncthreads();
     // 2. the nodes above the cut, deepest level first
@@ -93,16 +86,16 @@ fused_tree_kernel(FusedArgs a)
             const int k = idx / W, c = idx % W;
             if (c >= wu) continue;
             const int4 e = __ldg(a.tree_lev + beg + k);  // node, child_0, child_1
-            uint4 v = part[e.x * W + c];
-            if (e.y >= 0) v = V::op(part[e.y * W + c], v);
-            if (e.z >= 0) v = V::op(part[e.z * W + c], v);
+            T v = part[e.x * W + c];
+            if (e.y >= 0) v = U::op(part[e.y * W + c], v);
+            if (e.z >= 0) v = U::op(part[e.z * W + c], v);
             part[e.x * W + c] = v;
         }
         __syncthreads();
     }
     if (tid < wu) {
-        const uint4 v1 = part[a.tree_r1 * W + tid];
-        yrow[tid] = a.dual ? V::op(part[a.tree_r0 * W + tid], v1) : v1;
+        const T v1 = part[a.tree_r1 * W + tid];
+        yrow[tid] = a.dual ? U::op(part[a.tree_r0 * W + tid], v1) : v1;
     }
     __syncthreads();
     // 3. the result to every output
@@ -110,16 +103,30 @@ fused_tree_kernel(FusedArgs a)
 #pragma unroll 4
     for (int idx = tid; idx < nst; idx += kTreeThreads) {
         const int i = idx / W, c = idx % W;
-        if (c < wu) V::st(rank_ptr_w(a.y, i), u0 + c, yrow[c]);
+        if (c < wu) U::st(rank_ptr_w(a.y, i), u0 + c, yrow[c]);
+    }
+}
+
+template <class Op>
+__global__ void __launch_bounds__(kTreeThreads, 2)
+fused_tree_kernel(FusedArgs a)
+{
+    extern __shared__ uint4 smem[];
+    const int tid = threadIdx.x;
+    if (blockIdx.x < a.tree_tiles) {
+        const int64_t u0 = int64_t(blockIdx.x) * kTreeUnits;
+        tree_body<VecUnit<Op>>(a, u0, int(lmin(kTreeUnits, a.nvec - u0)), smem, smem + tid,
+                               kTreeThreads);
+    } else {  // ragged tail: the single elements after the 16-byte units
+        tree_body<OneUnit<Op>>(a, a.scalar_base, int(a.nscalar), smem, one_slots<Op>(smem, tid),
+                               one_slot_stride<Op>(kTreeThreads));
     }
 }
 
 size_t tree_smem(const Plan* P)
 {
-    const size_t walk = size_t(P->tree_slots) * kTreeThreads + size_t(P->tree_nseg) * kTreeUnits +
-                        kTreeUnits;
-    const size_t tail = size_t(P->max_depth + 2) * 32;  // the tail CTA's slots
-    return std::max(walk, tail) * sizeof(uint4);
+    return (size_t(P->tree_slots) * kTreeThreads + size_t(P->tree_nseg) * kTreeUnits +
+            kTreeUnits) * sizeof(uint4);
 }
 
 template <class Op>
