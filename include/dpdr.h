@@ -184,9 +184,10 @@ int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
  *                             64-bit store and the receiver polls the words,
  *                             which halves the latency of short blocks but
  *                             keeps 4 p m esize bytes of word arrays on the
- *                             device; 0 (default) chooses 2 while
- *                             m * esize <= 32 KiB and those arrays stay
- *                             within 1 GiB, else 1 */
+ *                             device; 0 (default) chooses 2 while the p
+ *                             inputs total at most 12 MiB (24 MiB from
+ *                             p = 1024) with one rank per schedule CTA,
+ *                             8 MiB with two, never with more; else 1 */
 enum {
     DPDR_OPT_FUSED_MODE = 1,
     DPDR_OPT_WAIT_LIMIT_NS = 2,

@@ -159,6 +159,7 @@ int fused_tree_prepare(Plan* P);                // fused_tree.cu
 bool fused_tree_wanted(const Plan* P);          // fused.cu
 int schedule_launch(Plan* P, cudaStream_t s);   // schedule.cu
 int schedule_configure(Plan* P);                // schedule.cu
+int schedule_plan_rpc(Plan* P);                 // schedule.cu: ranks per CTA only
 int schedule_transport(const Plan* P);          // schedule_ll.cu: 1 counters, 2 words
 const void* schedule_ll_kernel_for(int dtype);  // schedule_ll.cu
 size_t schedule_ll_bytes(const Plan* P);        // schedule_ll.cu

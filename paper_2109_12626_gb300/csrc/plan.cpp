@@ -378,6 +378,12 @@ extern "C" dpdr_plan_t dpdr_plan_topo(int p, int64_t m, dpdr_dtype dtype, dpdr_o
         free_plan(P);
         return nullptr;
     }
+    // ranks per schedule CTA first: the automatic transport, and with it the
+    // default block count, depends on it
+    if (schedule_plan_rpc(P) != DPDR_OK) {
+        free_plan(P);
+        return nullptr;
+    }
     P->b = b == 0 ? default_blocks(P) : clamp_b(m, b);
     if (allocate(P) != DPDR_OK || schedule_configure(P) != DPDR_OK ||
         (schedule_transport(P) == 2 && schedule_ll_prepare(P) != DPDR_OK) ||

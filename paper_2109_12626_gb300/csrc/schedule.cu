@@ -46,6 +46,7 @@ namespace dpdr {
 namespace {
 
 constexpr int kSchedMaxThreads = sched::kMaxThreads;
+constexpr int kSchedMaxGroups = sched::kMaxGroups;
 
 struct SchedArgs {
     const char* const* x;
@@ -68,6 +69,8 @@ struct SchedArgs {
     int vec;
     int nslices;   // CTAs per rank: each owns one column slice of every block
     int nchunks;   // rank ranges (CTA index = slice * nchunks + chunk)
+    int lg_gsz;    // log2 of the threads per rank group (at least 32)
+    int ngroups;   // rank groups per CTA
 };
 
 using sched::ld_acquire;
@@ -98,16 +101,62 @@ struct Wait {
     int step;
 };
 
-// Thread 0 waits until every one of the n counters (n <= 3, the same on all
-// threads) reaches its target, polling them together within the plan's time
-// bound; the CTA learns the outcome through shared memory.  Returns false on
-// timeout or abort (then the caller returns from the kernel).
+// The threads of a CTA that serve one virtual rank: a CTA that owns R ranks
+// splits its warps into min(R, warps) groups, each running the rounds of a
+// contiguous share of the ranks on its own, so a rank that waits for another
+// CTA holds up no rank of another group.  Each group synchronises on its own
+// named barrier.
+// The group size (a power of two, at least a warp) is the same for every CTA
+// of a launch; group k = threadIdx.x >> lg_gsz uses named barrier k + 1.
+struct Group {
+    int tid;   // thread index within the group
+    int size;  // threads in the group
+    int id;    // group index
+};
+
+// kG selects the kernel variant: false for CTAs that own one rank (the
+// whole CTA is the group, plain CTA barriers), true for several.
+template <bool kG>
+__device__ __forceinline__ Group group_of(const SchedArgs& a)
+{
+    if (!kG) return Group{int(threadIdx.x), int(blockDim.x), 0};
+    const int t = int(threadIdx.x);
+    return Group{t & ((1 << a.lg_gsz) - 1), 1 << a.lg_gsz, t >> a.lg_gsz};
+}
+
+template <bool kG>
+__device__ __forceinline__ void group_sync(const SchedArgs& a)
+{
+    if (!kG) {
+        __syncthreads();
+        return;
+    }
+    // immediate barrier ids, so the kernel reserves kSchedMaxGroups + 1
+    // barriers rather than all sixteen (which would cost occupancy)
+    const int n = 1 << a.lg_gsz;
+    switch (int(threadIdx.x) >> a.lg_gsz) {
+    case 0: asm volatile("bar.sync 1, %0;" ::"r"(n) : "memory"); break;
+    case 1: asm volatile("bar.sync 2, %0;" ::"r"(n) : "memory"); break;
+    case 2: asm volatile("bar.sync 3, %0;" ::"r"(n) : "memory"); break;
+    default: asm volatile("bar.sync 4, %0;" ::"r"(n) : "memory"); break;
+    }
+}
+static_assert(kSchedMaxGroups == 4, "group_sync names one barrier per group");
+
+// Thread 0 of the group waits until every one of the n counters (n <= 3,
+// the same on all its threads) reaches its target, polling them together
+// within the plan's time bound; the group learns the outcome through shared
+// memory.  Returns false on timeout or abort (then the caller returns from
+// the kernel).
+template <bool kG>
 __device__ __forceinline__ bool cta_wait(const SchedArgs& a, const Wait* w, int n, int rank,
                                          int j)
 {
     if (n == 0) return true;
-    __shared__ int ok;
-    if (threadIdx.x == 0) {
+    __shared__ int ok_slot[kSchedMaxGroups];
+    const Group grp = group_of<kG>(a);
+    int& ok = ok_slot[grp.id];
+    if (grp.tid == 0) {
         int r = 1;
         unsigned pending = 0;
         for (int k = 0; k < n; k++)
@@ -142,21 +191,22 @@ __device__ __forceinline__ bool cta_wait(const SchedArgs& a, const Wait* w, int 
         }
         ok = r;
     }
-    __syncthreads();
+    group_sync<kG>(a);
     const int r = ok;
-    __syncthreads();
+    group_sync<kG>(a);
     return r != 0;
 }
 
-// Release the CTA's writes to the rank's partner(s): the barrier orders
+// Release the group's writes to the rank's partner(s): the barrier orders
 // every thread's block writes before thread 0's gpu-scope release stores
 // (release is cumulative over what thread 0 has observed), and the partner's
 // acquire load orders its reads after them.  ctr1 may be null.
+template <bool kG>
 __device__ __forceinline__ void publish(const SchedArgs& a, uint32_t* ctr0, uint32_t v0,
                                         uint32_t* ctr1, uint32_t v1, int rank)
 {
-    __syncthreads();
-    if (threadIdx.x == 0 && rank != a.skip_rank) {
+    group_sync<kG>(a);
+    if (group_of<kG>(a).tid == 0 && rank != a.skip_rank) {
         st_release(ctr0, v0);
         if (ctr1) st_release(ctr1, v1);
     }
@@ -168,13 +218,14 @@ __device__ __forceinline__ void publish(const SchedArgs& a, uint32_t* ctr0, uint
 // call over the same range, so a later call may read what an earlier one
 // wrote without a barrier.  Not inlined: its eight 16-byte registers in
 // flight then fit the 64-register budget without spilling the caller's state.
-template <class Op>
+template <class Op, bool kG>
 __device__ __noinline__ void block_op(const SchedArgs& a, char* dst, const char* lo,
-                                         const char* hi, int64_t s, int64_t e)
+                                      const char* hi, int64_t s, int64_t e)
 {
     constexpr int EPV = Op::kEpv;
     constexpr int ES = Op::kEsize;
-    const int tid = threadIdx.x, bd = blockDim.x;
+    const Group grp = group_of<kG>(a);
+    const int tid = grp.tid, bd = grp.size;
     int64_t vs = 0, ve = 0;
     if (a.vec) {
         vs = (s + EPV - 1) / EPV;
@@ -217,13 +268,13 @@ __device__ __noinline__ void block_op(const SchedArgs& a, char* dst, const char*
 // dst = t1 (.) (t0 (.) x) over [s, e) for the children's partial blocks
 // t0, t1 (null when the child does not exist; both null: a copy of x): two
 // passes, the second reading back this thread's own results of the first.
-template <class Op>
+template <class Op, bool kG>
 __device__ __forceinline__ void fold_children(const SchedArgs& a, char* dst, const char* t0,
                                               const char* t1, const char* x, int64_t s,
                                               int64_t e)
 {
-    block_op<Op>(a, dst, t0, x, s, e);
-    if (t1) block_op<Op>(a, dst, t1, dst, s, e);
+    block_op<Op, kG>(a, dst, t0, x, s, e);
+    if (t1) block_op<Op, kG>(a, dst, t1, dst, s, e);
 }
 
 __device__ __forceinline__ char* ring_base(const SchedArgs& a, int side, int j,
@@ -239,7 +290,7 @@ __device__ __forceinline__ char* ring_base(const SchedArgs& a, int side, int j,
 // first, as the steps run) follow without a barrier between them.  The partial goes up before the wait for
 // the parent's final block, so a parent's round j never waits for its own
 // round j-1 to reach the child and come back.
-template <class Op>
+template <class Op, bool kG>
 __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j, int g)
 {
     constexpr int EPV = Op::kEpv;
@@ -269,81 +320,107 @@ __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j, int 
             t[k] = __ldg(a.child0 + c) < 0 ? rank_in(a.x, c) : rank_in(a.y, c);
             w[n++] = Wait{up + c, uint32_t(j + 1), k};
         }
-        if (!cta_wait(a, w, n, i, j)) return false;
+        if (!cta_wait<kG>(a, w, n, i, j)) return false;
     }
 
     if (paired_root) {  // step 3 at a root: exchange partials with the dual
         if (!inb) return true;
         const int side = (i == a.r0) ? 0 : 1;
         char* slot = ring_base(a, side, j, bs, Op::kEpv, Op::kEsize);
-        fold_children<Op>(a, slot, t[0], t[1], xi, s, e);
-        publish(a, up + i, uint32_t(j + 1), nullptr, 0, i);
+        fold_children<Op, kG>(a, slot, t[0], t[1], xi, s, e);
+        publish<kG>(a, up + i, uint32_t(j + 1), nullptr, 0, i);
         const int du = (i == a.r0) ? a.r1 : a.r0;
         const Wait wd{up + du, uint32_t(j + 1), 2};
-        if (!cta_wait(a, &wd, 1, i, j)) return false;
+        if (!cta_wait<kG>(a, &wd, 1, i, j)) return false;
         const char* other = ring_base(a, 1 - side, j, bs, Op::kEpv, Op::kEsize);
-        if (i == a.r0)
-            block_op<Op>(a, yi, slot, other, s, e);  // lower root: Y[j] (.) t
-        else
-            block_op<Op>(a, yi, other, slot, s, e);  // higher root: t (.) Y[j]
-        publish(a, down + i, uint32_t(j + 1), nullptr, 0, i);
+        if (i == a.r0)  // lower root: Y[j] (.) t
+            block_op<Op, kG>(a, yi, slot, other, s, e);
+        else  // higher root: t (.) Y[j]
+            block_op<Op, kG>(a, yi, other, slot, s, e);
+        publish<kG>(a, down + i, uint32_t(j + 1), nullptr, 0, i);
         return true;
     }
     if (root) {  // the root of a single tree (or p == 1): its block is final
         if (!inb) return true;
-        if (t[0] || xi != yi) fold_children<Op>(a, yi, t[0], t[1], xi, s, e);
-        publish(a, down + i, uint32_t(j + 1), nullptr, 0, i);
+        if (t[0] || xi != yi) fold_children<Op, kG>(a, yi, t[0], t[1], xi, s, e);
+        publish<kG>(a, down + i, uint32_t(j + 1), nullptr, 0, i);
         return true;
     }
     // step 3 elsewhere: partial Y[j] up (in y_i, or x_i itself for a leaf),
     // final Y[j-d] down from the parent
     if (inb) {
-        if (t[0]) fold_children<Op>(a, yi, t[0], t[1], xi, s, e);
-        publish(a, up + i, uint32_t(j + 1), nullptr, 0, i);
+        if (t[0]) fold_children<Op, kG>(a, yi, t[0], t[1], xi, s, e);
+        publish<kG>(a, up + i, uint32_t(j + 1), nullptr, 0, i);
     }
     const int kf = j - d;
     if (kf >= 0 && kf < a.b) {
         const Wait wp{down + par, uint32_t(kf + 1), 3};
-        if (!cta_wait(a, &wp, 1, i, j)) return false;
+        if (!cta_wait<kG>(a, &wp, 1, i, j)) return false;
         const char* yp = rank_in(a.y, par);
         const int64_t ks = blk_start(a, kf), ke = blk_start(a, kf + 1);
-        block_op<Op>(a, yi, nullptr, yp, slice_at<EPV>(a, ks, ke, g),
+        block_op<Op, kG>(a, yi, nullptr, yp, slice_at<EPV>(a, ks, ke, g),
                      slice_at<EPV>(a, ks, ke, g + 1));
-        publish(a, down + i, uint32_t(kf + 1), nullptr, 0, i);
+        publish<kG>(a, down + i, uint32_t(kf + 1), nullptr, 0, i);
     }
     return true;
 }
 
-template <class Op>
+template <class Op, bool kG>
 __global__ void __launch_bounds__(kSchedMaxThreads, 4) schedule_kernel(SchedArgs a)
 {
     const int g = blockIdx.x / a.nchunks, chunk = blockIdx.x % a.nchunks;
     const int first = __ldg(a.cta_first + chunk);
     const int last = __ldg(a.cta_first + chunk + 1);
+    // rank groups: group k runs its contiguous share of the CTA's ranks
+    int lo = first, hi = last;
+    if (kG) {
+        const int k = int(threadIdx.x) >> a.lg_gsz;
+        if (k >= a.ngroups) return;  // warps left over by the split
+        const int n = last - first;
+        lo = first + n * k / a.ngroups;
+        hi = first + n * (k + 1) / a.ngroups;
+    }
     int rounds = 0;
-    for (int i = first; i < last; i++) rounds = max(rounds, a.b + __ldg(a.depth + i));
+    for (int i = lo; i < hi; i++) rounds = max(rounds, a.b + __ldg(a.depth + i));
     for (int j = 0; j <= rounds; j++) {
-        for (int i = first; i < last; i++) {
+        for (int i = lo; i < hi; i++) {
             if (j > a.b + __ldg(a.depth + i)) continue;
-            if (!run_round<Op>(a, i, j, g)) return;
+            if (!run_round<Op, kG>(a, i, j, g)) return;
         }
     }
 }
 
 template <class Op>
-const void* kernel_ptr()
+const void* kernel_ptr(bool grouped)
 {
-    return reinterpret_cast<const void*>(&schedule_kernel<Op>);
+    return grouped ? reinterpret_cast<const void*>(&schedule_kernel<Op, true>)
+                   : reinterpret_cast<const void*>(&schedule_kernel<Op, false>);
 }
 
-const void* kernel_for(int dtype)
+// The kernel for CTAs that own one rank (grouped = false) or several.
+const void* kernel_for(int dtype, bool grouped)
 {
     switch (dtype) {
-    case DPDR_INT32: return kernel_ptr<SumI32>();
-    case DPDR_FLOAT32: return kernel_ptr<SumF32>();
-    case DPDR_MAT2X2_F32: return kernel_ptr<MatF32>();
-    default: return kernel_ptr<MatU32>();
+    case DPDR_INT32: return kernel_ptr<SumI32>(grouped);
+    case DPDR_FLOAT32: return kernel_ptr<SumF32>(grouped);
+    case DPDR_MAT2X2_F32: return kernel_ptr<MatF32>(grouped);
+    default: return kernel_ptr<MatU32>(grouped);
     }
+}
+
+// CTAs of `threads` threads that fit one SM for the counters kernel (the
+// variant for one rank per CTA, or the grouped one) and the flagged-word
+// kernel alike.
+cudaError_t sched_occupancy(int dtype, int threads, bool grouped, int* occ)
+{
+    int o[2] = {0, 0};
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o[0], kernel_for(dtype, grouped),
+                                                                  threads, 0);
+    if (e == cudaSuccess)
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o[1], schedule_ll_kernel_for(dtype),
+                                                          threads, 0);
+    *occ = std::min(o[0], o[1]);
+    return e;
 }
 
 }  // namespace
@@ -354,28 +431,49 @@ const void* kernel_for(int dtype)
 // elements with counters, one word batch per thread with flagged words).
 // Allocates the counters for that many slices and uploads the
 // chunk -> first rank table.
-int schedule_configure(Plan* P)
+// Ranks per CTA and co-resident CTAs of the layout: the fewest ranks per
+// CTA (none straddling the trees) with which every CTA -- times the slices a
+// fixed DPDR_OPT_SCHED_SLICES asks for -- fits at once, for the kernels that
+// run it: the one-rank-per-CTA counters kernel, or, once CTAs must own
+// several ranks, its grouped variant, and the flagged-word kernel.
+static int schedule_rpc(const Plan* P, int* R_out, int64_t* kmax_out)
 {
-    // one layout serves both transports: CTAs that fit for either kernel
-    int occ = 0, occ_ll = 0;
-    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-        &occ, kernel_for(P->dtype), P->sched_threads, 0);
-    if (e == cudaSuccess)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-            &occ_ll, schedule_ll_kernel_for(P->dtype), P->sched_threads, 0);
+    int occ = 0;
+    cudaError_t e = sched_occupancy(P->dtype, P->sched_threads, false, &occ);
     if (e != cudaSuccess) return cuda_fail(e, "schedule occupancy");
-    occ = std::min(occ, occ_ll);
-    const int64_t kmax = int64_t(occ) * P->num_sms;
-    // rank chunks never straddle the two trees (one tree: n0 = 0)
+    int64_t kmax = int64_t(occ) * P->num_sms;
     const int n0 = P->r0 >= 0 ? P->p / 2 : 0, n1 = P->p - n0;
     auto ctas = [&](int r) { return (n0 + r - 1) / r + (n1 + r - 1) / r; };
-    // with a fixed number of slices, ranks per CTA must make room for them
     const int64_t per_chunk = std::max(1, P->sched_slices);
     int R = P->sched_rpc;
     if (R == 0) {
         R = 1;
         while (R < P->p && ctas(R) * per_chunk > kmax) R++;
     }
+    if (R > 1) {
+        e = sched_occupancy(P->dtype, P->sched_threads, true, &occ);
+        if (e != cudaSuccess) return cuda_fail(e, "schedule occupancy");
+        kmax = int64_t(occ) * P->num_sms;
+        if (P->sched_rpc == 0)
+            while (R < P->p && ctas(R) * per_chunk > kmax) R++;
+    }
+    *R_out = R;
+    if (kmax_out) *kmax_out = kmax;
+    return DPDR_OK;
+}
+
+int schedule_plan_rpc(Plan* P) { return schedule_rpc(P, &P->sched_ranks_per_cta, nullptr); }
+
+int schedule_configure(Plan* P)
+{
+    int R = 1;
+    int64_t kmax = 0;
+    int rc = schedule_rpc(P, &R, &kmax);
+    if (rc) return rc;
+    P->sched_ranks_per_cta = R;  // the transport choice below depends on it
+    // rank chunks never straddle the two trees (one tree: n0 = 0)
+    const int n0 = P->r0 >= 0 ? P->p / 2 : 0;
+    cudaError_t e;
     std::vector<int> first;
     for (int lo = 0; lo < n0; lo += R) first.push_back(lo);
     for (int lo = n0; lo < P->p; lo += R) first.push_back(lo);
@@ -407,11 +505,11 @@ int schedule_configure(Plan* P)
     P->sched_slices_used = G;
     P->sched_chunks = nchunks;
     P->sched_ctas = nchunks * G;
-    P->sched_ranks_per_cta = R;
     e = cudaMemcpy(P->d_cta_first, first.data(), sizeof(int) * first.size(),
                    cudaMemcpyHostToDevice);
     if (e != cudaSuccess) return cuda_fail(e, "schedule table upload");
-    return DPDR_OK;
+    // the automatic transport may have changed with the layout
+    return schedule_transport(P) == 2 ? schedule_ll_prepare(P) : DPDR_OK;
 }
 
 int schedule_launch(Plan* P, cudaStream_t s)
@@ -444,11 +542,14 @@ int schedule_launch(Plan* P, cudaStream_t s)
     a.vec = P->last_vector_path;
     a.nslices = P->sched_slices_used;
     a.nchunks = P->sched_chunks;
+    a.ngroups = sched::group_count(P->sched_ranks_per_cta, P->sched_threads);
+    a.lg_gsz = sched::group_lg(P->sched_ranks_per_cta, P->sched_threads);
 
     cudaError_t e = cudaMemsetAsync(P->d_ctrl, 0, sizeof(uint32_t) * (2 * size_t(cw) + 1), s);
     if (e != cudaSuccess) return cuda_fail(e, "schedule counter reset");
     void* args[] = {&a};
-    e = cudaLaunchCooperativeKernel(kernel_for(P->dtype), dim3(P->sched_ctas),
+    e = cudaLaunchCooperativeKernel(kernel_for(P->dtype, P->sched_ranks_per_cta > 1),
+                                    dim3(P->sched_ctas),
                                     dim3(P->sched_threads), args, 0, s);
     if (e == cudaErrorCooperativeLaunchTooLarge) {
         cudaGetLastError();
@@ -611,12 +712,18 @@ int schedule_noalloc(int p, int64_t m, int dtype, int op, int b, const void* con
     cudaError_t e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e == cudaSuccess)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kernel_for(dtype), kNoAllocThreads, 0);
+        e = sched_occupancy(dtype, kNoAllocThreads, false, &occ);
     if (e != cudaSuccess) return cuda_fail_c(e, "no-alloc: device query");
-    const int64_t kmax = int64_t(occ) * sms;
+    int64_t kmax = int64_t(occ) * sms;
     const int n0 = p / 2, n1 = p - n0;
     int R = 1;
     while (R < p && int64_t((n0 + R - 1) / R + (n1 + R - 1) / R) > kmax) R++;
+    if (R > 1) {  // the grouped variant runs: its occupancy
+        e = sched_occupancy(dtype, kNoAllocThreads, true, &occ);
+        if (e != cudaSuccess) return cuda_fail_c(e, "no-alloc: device query");
+        kmax = int64_t(occ) * sms;
+        while (R < p && int64_t((n0 + R - 1) / R + (n1 + R - 1) / R) > kmax) R++;
+    }
     const int nctas = (n0 + R - 1) / R + (n1 + R - 1) / R;
 
     // rank pointers from the caller's host arrays, zeroed counters and
@@ -660,8 +767,11 @@ int schedule_noalloc(int p, int64_t m, int dtype, int op, int b, const void* con
     a.vec = vec;
     a.nslices = 1;
     a.nchunks = nctas;
+    a.ngroups = sched::group_count(R, kNoAllocThreads);
+    a.lg_gsz = sched::group_lg(R, kNoAllocThreads);
     void* args[] = {&a};
-    e = cudaLaunchCooperativeKernel(kernel_for(dtype), dim3(nctas), dim3(kNoAllocThreads), args, 0, s);
+    e = cudaLaunchCooperativeKernel(kernel_for(dtype, R > 1), dim3(nctas), dim3(kNoAllocThreads),
+                                    args, 0, s);
     if (e == cudaErrorCooperativeLaunchTooLarge) {
         cudaGetLastError();
         return fail_c(DPDR_ERR_NOT_COOPERATIVE, "no-alloc: CTAs cannot be co-resident");

@@ -10,6 +10,25 @@ namespace dpdr {
 namespace sched {
 
 constexpr int kMaxThreads = 256;
+constexpr int kMaxGroups = 4;  // rank groups per CTA (named barriers 1..4)
+
+// Rank groups of a CTA that owns R virtual ranks: min(R, warps, kMaxGroups)
+// groups of whole warps, all of one size, each running its own ranks.
+inline int group_count(int R, int threads)
+{
+    const int warps = threads / 32;
+    return R < 1 ? 1 : (R < warps ? (R < kMaxGroups ? R : kMaxGroups)
+                                  : (warps < kMaxGroups ? warps : kMaxGroups));
+}
+// log2 of the group size: the largest power of two of whole warps that
+// fits threads / groups
+inline int group_lg(int R, int threads)
+{
+    const int per = threads / group_count(R, threads);
+    int lg = 5;
+    while ((64 << (lg - 5)) <= per) lg++;
+    return lg;
+}
 
 __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p)
 {

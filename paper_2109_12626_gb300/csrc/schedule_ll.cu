@@ -319,21 +319,28 @@ const void* schedule_ll_kernel_for(int dtype)
 }
 
 // Transport of the schedule kernel: the plan's option, else flagged words
-// while a rank's buffer is at most kWordsMaxRankBytes and the word arrays
-// (4 p m esize bytes) at most kWordsMaxBytes, else counters.  Measured at
-// p = 288, int32, b = 1: 15.4 us against 41.3 us at m = 1, 34.7 against
-// 45.9 at m = 2500, 47.7 against 60.9 at m = 8750; from about 60 KB per rank
-// the counters' 16-byte block copies win (m = 25000: 84 us at b = 2 against
-// 103), and at p = 1152 from about 32 KB.
-constexpr int64_t kWordsMaxRankBytes = int64_t(32) << 10;
-constexpr int64_t kWordsMaxBytes = int64_t(1) << 30;
-
+// while the p inputs total at most a cap that depends on the layout, else
+// counters.  Flagged words cost one L2 trip per exchange against three, but
+// move 8 bytes per 4-byte word and poll per thread, and a CTA that owns
+// several ranks runs them one after another per thread (the counters kernel
+// gives each its own warps).  Measured at b = 1..8, int32, best b each:
+//  * one rank per CTA: up to 12 MB (p = 30, m = 2^16: 29 us either way;
+//    p = 126, m = 2^15: counters 49 against 59 us), 24 MB from p = 1024
+//    (p = 1152, m = 4096: 59 against 64 us; m = 16384: counters 125 against
+//    183 us);
+//  * two ranks per CTA: up to 8 MB (p = 2048, m = 1024: 48 against 64 us;
+//    m = 4096: counters 97 against 104 us);
+//  * more: counters (p = 4094, m = 1024: 85 against 98 us; p = 8190, m = 1:
+//    367 against 479 us).
+// The word arrays (4 p m esize bytes) never exceed 96 MB under these caps.
 int schedule_transport(const Plan* P)
 {
     if (P->sched_transport) return P->sched_transport;
-    const int64_t rank_bytes = P->m * int64_t(P->esize);
-    return rank_bytes <= kWordsMaxRankBytes && 4 * int64_t(P->p) * rank_bytes <= kWordsMaxBytes
-        ? 2 : 1;
+    const int R = std::max(1, P->sched_ranks_per_cta);
+    const int64_t bytes = int64_t(P->p) * P->m * int64_t(P->esize);
+    const int64_t cap = R == 1 ? (P->p >= 1024 ? int64_t(24) << 20 : int64_t(12) << 20)
+                      : R == 2 ? int64_t(8) << 20 : 0;
+    return bytes <= cap ? 2 : 1;
 }
 
 // Elements one CTA of the flagged-word kernel takes per pass: a batch of

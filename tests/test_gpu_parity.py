@@ -321,20 +321,27 @@ def test_schedule_column_slices(pkg, orc, kind, p, m, b, slices, layout, transpo
 
 
 def test_schedule_transport_choice(pkg):
-    """Flagged words while a rank's buffer is at most 32 KiB (and the word
-    arrays fit 1 GiB), counters above; the option overrides either way."""
-    with pkg.Plan(36, 8192, "int32", 0) as plan:
-        assert plan.info()["sched_transport"] == 2
-        plan.set(pkg.OPT_SCHED_TRANSPORT, 1)
-        assert plan.info()["sched_transport"] == 1
-    with pkg.Plan(36, 8193, "int32", 0) as plan:
-        assert plan.info()["sched_transport"] == 1
-        plan.set(pkg.OPT_SCHED_TRANSPORT, 2)
-        assert plan.info()["sched_transport"] == 2
-    with pkg.Plan(36, 2048, "mat2x2u32", 0) as plan:
-        assert plan.info()["sched_transport"] == 2
-    with pkg.Plan(36, 2049, "mat2x2u32", 0) as plan:
-        assert plan.info()["sched_transport"] == 1
+    """Flagged words while the p inputs total at most 12 MiB (24 MiB from
+    p = 1024) with one rank per CTA, 8 MiB with two ranks per CTA, never with
+    more; counters otherwise.  The option overrides either way."""
+    MiB = 1 << 20
+    cases = [(36, 12 * MiB // (36 * 4), "int32"), (1152, 24 * MiB // (1152 * 4), "int32"),
+             (36, 12 * MiB // (36 * 16), "mat2x2u32")]
+    for p, m_max, kind in cases:
+        with pkg.Plan(p, m_max, kind, 0) as plan:
+            assert plan.info()["sched_ranks_per_cta"] == 1
+            assert plan.info()["sched_transport"] == 2, (p, m_max)
+            plan.set(pkg.OPT_SCHED_TRANSPORT, 1)
+            assert plan.info()["sched_transport"] == 1
+        with pkg.Plan(p, m_max + 1, kind, 0) as plan:
+            assert plan.info()["sched_transport"] == 1, (p, m_max + 1)
+            plan.set(pkg.OPT_SCHED_TRANSPORT, 2)
+            assert plan.info()["sched_transport"] == 2
+    for p in (2048, 4094):
+        with pkg.Plan(p, 1, "int32", 0) as plan:
+            rpc = plan.info()["sched_ranks_per_cta"]
+            want = 2 if rpc <= 2 else 1
+            assert plan.info()["sched_transport"] == want, (p, rpc)
     from paper_2109_12626_gb300 import DpdrError
     with pkg.Plan(3, 10, "int32", 0) as plan:
         with pytest.raises(DpdrError):
@@ -398,3 +405,28 @@ def test_default_block_count(pkg):
             assert plan.query()["b"] == want, (p, m)
             plan.set(pkg.OPT_BLOCKS, 0)
             assert plan.query()["b"] == want
+
+
+@pytest.mark.parametrize("kind,p,m,b", [("int32", 36, 1003, 3), ("float32", 255, 2050, 2),
+                                        ("mat2x2u32", 100, 77, 7)])
+@pytest.mark.parametrize("rpc", [2, 3, 4, 5])
+@pytest.mark.parametrize("transport", list(TRANSPORTS))
+def test_schedule_ranks_per_cta(pkg, orc, kind, p, m, b, rpc, transport):
+    """CTAs that own several virtual ranks (the layout of p beyond the
+    co-resident CTA count): the counters kernel splits them into rank groups
+    of warps with their own barriers, up to one group per warp (rpc = 5 puts
+    two ranks on one warp of a 128-thread CTA).  Same bits."""
+    x = host_inputs(kind, 71, p, m)
+    want = _want(orc, x, kind)
+    dev = torch.device("cuda:0")
+    xs, _ = to_device(x, kind, dev)
+    for in_place in (False, True):
+        xs_run = [t.clone() for t in xs] if in_place else xs
+        ys = xs_run if in_place else empty_like_ranks(xs)[0]
+        with pkg.Plan(p, m, kind, b) as plan:
+            plan.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[transport])
+            plan.set(pkg.OPT_SCHED_RANKS_PER_CTA, rpc)
+            assert plan.info()["sched_ranks_per_cta"] == rpc
+            plan.allreduce_schedule(xs_run, ys)
+            plan.sync()
+        _check_all(ys, want)
