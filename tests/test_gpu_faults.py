@@ -23,7 +23,7 @@ def pkg():
     return P
 
 
-@pytest.mark.parametrize("p,skip", [(7, 0), (7, 6), (36, 17), (1152, 700)])
+@pytest.mark.parametrize("p,skip", [(7, 0), (7, 6), (36, 17), (1152, 700), (4094, 3000)])
 @pytest.mark.parametrize("transport", [1, 2], ids=["counters", "words"])
 def test_silent_rank_times_out_and_recovers(pkg, orc, p, skip, transport):
     from paper_2109_12626_gb300 import DpdrError

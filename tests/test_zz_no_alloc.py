@@ -37,8 +37,10 @@ def _call_noalloc(N, p, m, dt, op, b, xs, ys):
     return L.dpdr_allreduce_schedule_noalloc(p, m, dt, op, b, X, Y, stream)
 
 
+# p = 3000 puts several ranks on each CTA (rank groups)
 CASES = [("int32", 7, 1000, 4), ("mat2x2u32", 36, 4099, 16),
-         ("float32", 1152, 4099, 0), ("float32", 32, 65541, 64), ("int32", 2, 3, 3)]
+         ("float32", 1152, 4099, 0), ("float32", 32, 65541, 64), ("int32", 2, 3, 3),
+         ("int32", 3000, 257, 2)]
 
 
 @pytest.mark.parametrize("kind,p,m,b", CASES)
