@@ -39,6 +39,10 @@ CASES = [
     ("p3_m801_f32", "float32", 9, 3, 801, {}, [2]),
     ("p32_m803_int32", "int32", 9, 32, 803, {}, [3]),
     ("p1152_m1021_f32", "float32", 9, 1152, 1021, {}, [2]),
+    # near the largest p the allocation-free entry point takes (8192): deep
+    # trees (depth 11), eight ranks per schedule CTA, a 131 KB tile row
+    ("p8190_m33_int32", "int32", 10, 8190, 33, dict(lo=-1000, hi=1000), [1, 2]),
+    ("p8190_m7_f32", "float32", 10, 8190, 7, dict(sigma=1.0), [1]),
 ]
 
 
@@ -430,3 +434,20 @@ def test_schedule_ranks_per_cta(pkg, orc, kind, p, m, b, rpc, transport):
             plan.allreduce_schedule(xs_run, ys)
             plan.sync()
         _check_all(ys, want)
+
+
+@pytest.mark.parametrize("run", RUNS)
+def test_int32_sums_wrap(pkg, orc, run):
+    """Full-range int32 inputs: the sums overflow and wrap modulo 2^32 (two's
+    complement), the same on every path as in the oracle."""
+    from paper_2109_12626_gb300 import inputs as I
+    p, m = 1152, 1027
+    x = np.stack([I.words_u32(12, i, m, 2)[:, 0].numpy() for i in range(p)])
+    assert np.abs(x.astype(np.int64)).max() > (1 << 30)
+    want = _want(orc, x, "int32")
+    xs, _ = to_device(x, "int32", torch.device("cuda:0"))
+    ys, _ = empty_like_ranks(xs)
+    with pkg.Plan(p, m, "int32", 3) as plan:
+        _run(pkg, plan, run, xs, ys)
+        plan.sync()
+    _check_all(ys, want)
