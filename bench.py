@@ -589,7 +589,7 @@ def main(argv=None) -> int:
         os.sched_setaffinity(0, saved)
 
     cpu = None
-    if rank == 0 and not args.no_cpu:
+    if rank == 0 and world == 1 and not args.no_cpu:  # the CPU baseline: N = 1 only
         gbs, sample, _ = cpu_sample(w, args.cpu_seconds)
         cpu = {"value": round(gbs, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
                "sample": sample}
