@@ -216,9 +216,12 @@ def kernel_source_hash(kernel: str) -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(kernel: str, wname: str, units: int) -> float | None:
+def profiled_traffic(kernel: str, wname: str, units: int,
+                     block: int | None = None) -> float | None:
     """DRAM bytes per launch from the committed ncu summary, scaled to the
-    units of this launch; None if the kernel changed since the capture."""
+    units of this launch; None if the kernel changed since the capture, or
+    (schedule kernel) if the capture's pipeline block size was not within
+    5 % of this run's, since the traffic depends on it."""
     path = os.path.join(ROOT, "profiles", "traffic.json")  # ncu figures, not code
     try:
         with open(path) as f:
@@ -226,6 +229,9 @@ def profiled_traffic(kernel: str, wname: str, units: int) -> float | None:
     except (OSError, KeyError, ValueError):
         return None
     if rec.get("source_hash") != kernel_source_hash(kernel):
+        return None
+    want = rec.get("block_elems")
+    if want is not None and (block is None or abs(block - want) > 0.05 * want):
         return None
     return float(rec["bytes_per_unit"]) * units
 
@@ -618,7 +624,8 @@ def main(argv=None) -> int:
         "roofline": {"bound": "hbm", "kernel": layout, "achieved": round(achieved, 1), "peak": peak,
                      "unit": "GB/s", "frac": round(achieved / peak, 4),
                      "peak_kind": peak_kind + " copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
-                     "traffic": profiled_traffic(layout, args.workload, units),
+                     "traffic": profiled_traffic(layout, args.workload, units,
+                                                 -(-m // max(1, info["b"]))),
                      "kernel_ms": round(avg_launch, 4)},
         "cpu_baseline": cpu,
         "e2e": e2e,

@@ -70,9 +70,13 @@ def test_profiled_traffic_tracks_the_kernel_source():
     rec = json.load(open(os.path.join(ROOT, "profiles", "traffic.json")))
     for kernel, table in rec.items():
         for wname, r in table.items():
-            got = bench.profiled_traffic(kernel, wname, 1000)
+            blk = r.get("block_elems")
+            got = bench.profiled_traffic(kernel, wname, 1000, blk)
             if r["source_hash"] == bench.kernel_source_hash(kernel):
                 assert got == pytest.approx(1000 * r["bytes_per_unit"])
+                if blk is not None:  # the schedule kernel's traffic depends on the block size
+                    assert bench.profiled_traffic(kernel, wname, 1000, 2 * blk) is None
+                    assert bench.profiled_traffic(kernel, wname, 1000, None) is None
             else:
                 assert got is None  # stale counters are not reported
 
