@@ -362,11 +362,41 @@ def _timed(fn, reps, stream, graph=False):
     return a.elapsed_time(z) / reps * 1e-3
 
 
+def _timed_reps(fn, reps):
+    """Per-call times (seconds) of reps replays of a CUDA graph holding one
+    call, each bracketed by its own events, after three untimed replays."""
+    import torch
+    for _ in range(2):
+        fn()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        fn()
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(reps)]
+    for a, z in ev:
+        a.record()
+        g.replay()
+        z.record()
+    torch.cuda.synchronize()
+    return [a.elapsed_time(z) * 1e-3 for a, z in ev]
+
+
+def _stats(ts):
+    """mean, min (the paper's convention: the best of the measurement
+    rounds) and median, in microseconds."""
+    return {"us": round(statistics.fmean(ts) * 1e6, 2), "us_min": round(min(ts) * 1e6, 2),
+            "us_median": round(statistics.median(ts) * 1e6, 2)}
+
+
 def run_sweep(args, w) -> int:
     """--sweep m: every m = 2^0 .. 2^k of the workload, fused kernel (its
     automatic layout) and schedule kernel (its automatic transport) at the
-    block-count rule, both timed as CUDA-graph replays so host launch
-    overhead is excluded.  --sweep b: the schedule
+    block-count rule, both timed as CUDA-graph replays of one call each (host
+    launch overhead excluded): mean, min and median over the replays.  --sweep b: the schedule
     kernel's time against b at one m, with the Sec. 1.2 cost model fitted.
     One JSON line per point, then a summary line."""
     import torch
@@ -388,19 +418,20 @@ def run_sweep(args, w) -> int:
             with pkg.Plan(p, m, kind, b0, topology=args.topology) as plan:
                 plan.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[args.transport])
                 bd = plan.bind(xs, ys)
-                t = _timed(lambda: bd.allreduce(), 20, None, graph=True)
+                st = _stats(_timed_reps(lambda: bd.allreduce(), 20))
                 info = plan.info()
-                rec["fused"] = {"us": round(t * 1e6, 2), "gbs": round(2 * p * m * es / t / 1e9, 2),
-                                "layout": LAYOUTS[info["auto_mode"]],
-                                "split_depth": info["split_depth"] if info["auto_mode"] == 3 else None}
-                t = _timed(lambda: bd.allreduce_schedule(), 3 if m >= (1 << 20) else 10, None,
-                           graph=True)
+                rec["fused"] = dict(st, gbs=round(2 * p * m * es / (st["us"] * 1e-6) / 1e9, 2),
+                                    layout=LAYOUTS[info["auto_mode"]],
+                                    split_depth=info["split_depth"] if info["auto_mode"] == 3
+                                    else None)
+                st = _stats(_timed_reps(lambda: bd.allreduce_schedule(),
+                                        5 if m >= (1 << 20) else 20))
                 plan.sync()
-                rec["schedule"] = {"b": info["b"], "us": round(t * 1e6, 2),
-                                   "gbs": round(2 * p * m * es / t / 1e9, 2),
-                                   "slices": plan.info()["sched_slices"],
-                                   "transport": ("counters", "words")[
-                                       info["sched_transport"] - 1]}
+                rec["schedule"] = dict(st, b=info["b"],
+                                       gbs=round(2 * p * m * es / (st["us"] * 1e-6) / 1e9, 2),
+                                       slices=plan.info()["sched_slices"],
+                                       transport=("counters", "words")[
+                                           info["sched_transport"] - 1])
             print(json.dumps(rec), flush=True)
             del xs, ys
             torch.cuda.empty_cache()
