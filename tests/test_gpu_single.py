@@ -1,7 +1,7 @@
 """GPU parity for the one-tree topology (Sec. 1.2's single doubly pipelined
-tree): every fused layout and the schedule kernel, bit for bit against the
-oracle's one-tree fold, whose float32 bracketing differs from the dual
-trees'."""
+tree): every fused layout and the schedule kernel (both transports, column
+slices, several ranks per CTA), bit for bit against the oracle's one-tree
+fold, whose float32 bracketing differs from the dual trees'."""
 import numpy as np
 import pytest
 import torch
@@ -31,7 +31,8 @@ def _want(orc, x, kind):
 
 
 @pytest.mark.parametrize("kind,p,m", CASES)
-@pytest.mark.parametrize("run", ["stream", "tile", "split", "bulk", "schedule", "schedule_slices"])
+@pytest.mark.parametrize("run", ["stream", "tile", "split", "bulk", "tree", "schedule_counters",
+                                 "schedule_words", "schedule_slices", "schedule_groups"])
 def test_single_tree_parity(pkg, orc, kind, p, m, run):
     x = host_inputs(kind, 71, p, m)
     want = _want(orc, x, kind)
@@ -43,9 +44,13 @@ def test_single_tree_parity(pkg, orc, kind, p, m, run):
         if run.startswith("schedule"):
             if run == "schedule_slices":
                 plan.set(pkg.OPT_SCHED_SLICES, 3)
+            if run == "schedule_groups":
+                plan.set(pkg.OPT_SCHED_RANKS_PER_CTA, min(p, 3))
+            if run in ("schedule_counters", "schedule_words"):
+                plan.set(pkg.OPT_SCHED_TRANSPORT, 1 if run == "schedule_counters" else 2)
             plan.allreduce_schedule(xs, ys)
         else:
-            mode = {"stream": 1, "tile": 2, "split": 3, "bulk": 4}[run]
+            mode = {"stream": 1, "tile": 2, "split": 3, "bulk": 4, "tree": 5}[run]
             if mode == 3 and p < 2:
                 pytest.skip("split layout needs p >= 2")
             plan.set(pkg.OPT_FUSED_MODE, mode)
