@@ -249,10 +249,12 @@ int dpdr_allreduce_schedule(dpdr_plan_t plan, const void* const* x,
  * of p pointers).  Two paths:
  *   direct  when the GPU can address every host buffer (pinned memory, or
  *           pageable memory on systems whose GPU uses the CPU page tables,
- *           such as Grace with NVLink-C2C): one launch of the column-
- *           streaming fused kernel loads the inputs from host memory and
- *           stores the result to host memory, both link directions at once;
- *           x_dev and y_dev are not used and may be NULL.
+ *           such as Grace with NVLink-C2C): one launch of the fused kernel
+ *           (the layout DPDR_OPT_FUSED_MODE names, else the hierarchical
+ *           tile, or column streaming below 1 MiB of inputs and above 4 GiB
+ *           at p < 64) loads the inputs from host memory and stores the result
+ *           to host memory, both link directions at once; x_dev and y_dev
+ *           are not used and may be NULL.
  *   copy    otherwise: the columns are cut into chunks (about 1 GB of rank
  *           data each) that flow through a pipeline -- copies into the
  *           device buffers x_dev[i] on one plan-owned stream, the kernel on

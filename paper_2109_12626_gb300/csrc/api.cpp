@@ -227,13 +227,28 @@ extern "C" int dpdr_allreduce_host(dpdr_plan_t h, const void* const* x_host,
     for (int i = 0; i < P->p; i++)
         if (!x_host[i] || !y_host[i]) return fail(DPDR_ERR_INVALID, "NULL host buffer");
     if (P->m == 0) return DPDR_OK;
-    // direct: the streaming layout loads the inputs from host memory and
-    // stores the result to host memory, both link directions at once
+    // direct: one launch loads the inputs from host memory and stores the
+    // result to host memory, the link carrying both directions at once.  The
+    // layout DPDR_OPT_FUSED_MODE names, else the hierarchical tile, whose
+    // CTAs read all their columns, then write them, and drift out of phase
+    // with each other (p = 1152, m = 2^20: 297 GB/s against 230 for column
+    // streaming, whose threads read and write in long lockstep phases at
+    // large p; p = 288, m = 2^22: 339 against 270; p = 36, 2x2 matrices,
+    // m = 2^16: 315 against 213); column streaming below 1 MiB of inputs,
+    // where one phase per thread has the least latency (p = 7, m = 1000:
+    // 4.5 against 3.7 GB/s), and above 4 GiB at p < 64, where its 4 KB row
+    // pieces per CTA suit the link better (p = 32, m = 2^27: 333 against
+    // 318; m = 2^25: 320 against 343)
     if (P->host_path != 1 && resolve_direct(P, x_host, y_host)) {
         int rc = prepare(P, P->direct_dx.data(), P->direct_dy.data(), s);
         if (rc) return rc;
+        const int64_t bytes = int64_t(P->p) * P->m * int64_t(P->esize);
+        const bool stream = bytes < (int64_t(1) << 20) ||
+                            (P->p < 64 && bytes > (int64_t(4) << 30));
+        const int mode = P->fused_mode ? P->fused_mode : stream ? 1 : 5;
+        if (mode == 5 && (rc = fused_tree_prepare(P)) != DPDR_OK) return rc;
         P->last_host_path = 2;
-        return fused_launch_cols(P, P->d_x, P->d_y, P->m, P->last_vector_path != 0, s, 1);
+        return fused_launch_cols(P, P->d_x, P->d_y, P->m, P->last_vector_path != 0, s, mode);
     }
     if (P->host_path == 2)
         return fail(DPDR_ERR_INVALID, "dpdr_allreduce_host: host buffers not addressable by the GPU");
