@@ -1,4 +1,4 @@
-// dpdr_internal.h -- plan layout shared by the host code and the two kernel
+// dpdr_internal.h -- plan layout shared by the host code and the kernel
 // launchers of the library (not part of the public ABI).
 #pragma once
 
