@@ -156,7 +156,6 @@ int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t m
 int fused_auto_mode(const Plan* P);             // fused.cu
 int fused_split_prepare(Plan* P, bool force, int depth);  // fused.cu
 int fused_tree_prepare(Plan* P);                // fused_tree.cu
-bool fused_tree_wanted(const Plan* P);          // fused.cu
 int schedule_launch(Plan* P, cudaStream_t s);   // schedule.cu
 int schedule_configure(Plan* P);                // schedule.cu
 int schedule_plan_rpc(Plan* P);                 // schedule.cu: ranks per CTA only

@@ -61,10 +61,6 @@ int fused_auto_mode(const Plan* P)
     return P->split_ready ? 3 : 1;
 }
 
-// Whether the automatic choice can be the hierarchical tile (then the plan
-// prepares its tables up front).
-bool fused_tree_wanted(const Plan* P) { return tree_preferred(P); }
-
 // Whether the automatic choice can be the split layout (then the plan
 // prepares it up front).
 static bool split_wanted(const Plan* P)

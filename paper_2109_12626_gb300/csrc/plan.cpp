@@ -387,7 +387,7 @@ extern "C" dpdr_plan_t dpdr_plan_topo(int p, int64_t m, dpdr_dtype dtype, dpdr_o
     P->b = b == 0 ? default_blocks(P) : clamp_b(m, b);
     if (allocate(P) != DPDR_OK || schedule_configure(P) != DPDR_OK ||
         (schedule_transport(P) == 2 && schedule_ll_prepare(P) != DPDR_OK) ||
-        (fused_tree_wanted(P) && fused_tree_prepare(P) != DPDR_OK) ||
+        fused_tree_prepare(P) != DPDR_OK ||  // small; the host path may use it
         fused_split_prepare(P, false, P->split_depth) != DPDR_OK) {
         free_plan(P);
         return nullptr;
