@@ -107,3 +107,19 @@ def test_single_tree_matches_oracle(native, orc, p):
     o = orc.trees(p, orc.SINGLE)
     for k in ("parent", "child0", "child1", "dual", "depth"):
         assert np.array_equal(a[k], o[k]), k
+
+
+def test_header_is_iso_c99_and_a_c_program_links(native, tmp_path):
+    """The boundary stands without Python: include/dpdr.h compiles as strict
+    C99, and a plain C program that calls every run entry point links
+    against libdpdr.so and the CUDA runtime (it runs in the GPU tests)."""
+    import c_build
+    if c_build.cc() is None:
+        pytest.skip("no C compiler")
+    r = c_build.compile_header_as_c(str(tmp_path))
+    assert r.returncode == 0, r.stderr
+    if not os.path.exists(os.path.join(c_build.CUDA, "include", "cuda_runtime_api.h")):
+        pytest.skip("no CUDA headers")
+    r, exe = c_build.build_program(str(tmp_path))
+    assert r.returncode == 0, r.stderr
+    assert os.path.exists(exe)
