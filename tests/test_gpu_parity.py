@@ -451,3 +451,32 @@ def test_int32_sums_wrap(pkg, orc, run):
         _run(pkg, plan, run, xs, ys)
         plan.sync()
     _check_all(ys, want)
+
+
+@pytest.mark.parametrize("run", ["fused_auto", "fused_stream", "fused_tree", "fused_split",
+                                 "schedule_auto"])
+def test_very_many_ranks(pkg, orc, run):
+    """p = 65535 ranks of 5 elements: trees of depth 15, about 54 ranks per
+    schedule CTA (4 rank groups), the tile layout out of reach (a tile row
+    would exceed shared memory).  Every path still gives the oracle's bits."""
+    kind, p, m = "float32", 65535, 5
+    # one seeded draw for all ranks (the per-rank generator takes ~30 s here);
+    # both sides get the same array
+    x = np.random.default_rng(81).standard_normal((p, m)).astype(np.float32)
+    want = _want(orc, x, kind)
+    dev = torch.device("cuda:0")
+    xs = list(torch.from_numpy(x).to(dev).unbind(0))  # p views of one allocation
+    ys = list(torch.full((p, m), -3.0, device=dev).unbind(0))
+    with pkg.Plan(p, m, kind, 0) as plan:
+        if run == "schedule_auto":
+            assert plan.info()["sched_ranks_per_cta"] > 4
+            plan.allreduce_schedule(xs, ys)
+        else:
+            mode = {"fused_auto": 0, "fused_stream": 1, "fused_tree": 5, "fused_split": 3}[run]
+            if mode:
+                plan.set(pkg.OPT_FUSED_MODE, mode)
+            plan.allreduce(xs, ys)
+        plan.sync()
+    got = torch.stack(ys).cpu().numpy().view(np.int32)
+    bad = np.nonzero((got != want.reshape(1, m)).any(axis=1))[0]
+    assert bad.size == 0, "%d ranks differ, first %d" % (bad.size, bad[0] if bad.size else -1)
