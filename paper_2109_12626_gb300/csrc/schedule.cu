@@ -29,14 +29,16 @@
 // A virtual rank is served by a group of nslices CTAs, one per column slice
 // of every pipeline block; slices are independent copies of the schedule
 // (their own counters), since (.) acts column by column.  CTAs own
-// contiguous rank ranges that never straddle the two trees and run
-// their ranks in increasing order inside each round.  Every wait is then on
-// a lower rank of the same round, on an earlier round, or (r0 only) on the
-// dual r1 whose partial depends on tree 1 alone, so with all CTAs resident
-// (cooperative launch) the schedule cannot deadlock.  With one tree (no
-// dual) the root's partial block j is final and is published down at once.  Each wait is bounded
-// in time; an expired wait records {rank, round, step} in the plan's error
-// word, raises an abort flag that ends every other wait, and returns.
+// contiguous rank ranges that never straddle the two trees; a CTA that owns
+// several splits its warps into rank groups (see Group below), and each
+// group runs its ranks in increasing order inside each round.  Every wait is
+// then on a lower rank of the same round, on an earlier round, or (r0 only)
+// on the dual r1 whose partial depends on tree 1 alone, so with all CTAs
+// resident (cooperative launch) the schedule cannot deadlock.  With one tree
+// (no dual) the root's partial block j is final and is published down at
+// once.  Each wait is bounded in time; an expired wait records {rank, round,
+// step} in the plan's error word, raises an abort flag that ends every other
+// wait, and returns.
 #include <algorithm>
 #include <mutex>
 
