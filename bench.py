@@ -208,11 +208,22 @@ def measured_peak_gbs() -> tuple[float, str]:
         return 6800.0, "fallback"
 
 
+def _code_only(text: str) -> str:
+    """C++ source without comments and blank space, so that editing a comment
+    does not mark measured counters stale (string literals here hold no
+    comment markers)."""
+    import re
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return " ".join(text.split())
+
+
 def kernel_source_hash(kernel: str) -> str:
+    """Hash of the code (comments and spacing aside) of a layout's sources."""
     h = hashlib.sha256()
     for f in KERNEL_SOURCES[kernel] + ("ops.cuh",):
-        with open(os.path.join(ROOT, "paper_2109_12626_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2109_12626_gb300", "csrc", f)) as fh:
+            h.update(_code_only(fh.read()).encode())
     return h.hexdigest()[:16]
 
 
