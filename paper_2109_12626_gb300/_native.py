@@ -183,13 +183,13 @@ class Plan:
         return out
 
     def info(self) -> dict:
-        v = np.zeros(16, np.int64)
-        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), 16),
+        v = np.zeros(17, np.int64)
+        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), 17),
                "dpdr_plan_info")
         keys = ("p", "m", "b", "max_depth", "auto_mode", "sched_ctas",
                 "sched_ranks_per_cta", "scratch_bytes", "vector_path",
                 "split_depth", "split_subtrees", "split_group", "sched_slices",
-                "topology", "host_path", "sched_transport")
+                "topology", "host_path", "sched_transport", "tree_width")
         return {k: int(x) for k, x in zip(keys, v)}
 
     def set(self, key: int, value: int) -> None:

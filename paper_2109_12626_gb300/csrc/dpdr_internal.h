@@ -89,7 +89,8 @@ struct Plan {
     bool staged_pending = false;     // d_x / d_y hold last_x / last_y
 
     // dynamic shared memory already granted to the fused kernels of this
-    // plan's element type (stream, tile), so launches skip the attribute call
+    // plan's element type (stream, tile, split, bulk, hierarchical tile), so
+    // launches skip the attribute call; the limits themselves only ever rise
     int smem_attr[5] = {48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024};
 
     // split layout of the fused kernel (fused.cu): subtrees at depth split_s
@@ -106,6 +107,7 @@ struct Plan {
     // (subtrees at depth tree_s, then nodes above the cut) and level table
     bool tree_ready = false;
     int tree_s = 0, tree_nseg = 0, tree_nlev = 0, tree_slots = 0, tree_r0 = -1, tree_r1 = 0;
+    int tree_width = 0;              // column units per CTA
     char* d_tree = nullptr;          // own allocation
     size_t d_tree_bytes = 0;
     int2* d_tree_seg = nullptr;

@@ -1,9 +1,32 @@
 // fused.cu -- layout choice and launch of the fused bandwidth kernel
 // (dpdr_allreduce); the layouts themselves live in fused_stream.cu,
 // fused_tile.cu, fused_split.cu and fused_bulk.cu (see fused_common.cuh).
+#include <map>
+#include <mutex>
+#include <utility>
+
 #include "fused_common.cuh"
 
 namespace dpdr {
+
+int fused::grant_smem(const void* fn, size_t bytes, int* granted, const char* what)
+{
+    if (int(bytes) <= *granted) return DPDR_OK;
+    static std::mutex mu;
+    static std::map<std::pair<int, const void*>, int> limit;  // (device, kernel) -> bytes
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, what);
+    std::lock_guard<std::mutex> lock(mu);
+    int& cur = limit[std::make_pair(dev, fn)];
+    if (int(bytes) > cur) {
+        e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, int(bytes));
+        if (e != cudaSuccess) return cuda_fail(e, what);
+        cur = int(bytes);
+    }
+    *granted = int(bytes);
+    return DPDR_OK;
+}
 
 using fused::FusedArgs;
 using fused::kBulkTile;
@@ -14,15 +37,18 @@ static int64_t stream_target(const Plan* P) { return int64_t(P->num_sms) * 1024;
 
 // Layout choice, from layout sweeps measured on GB300 (int32, p = 128 ...
 // 4096, m = 2^10 ... 2^20, warm and cold L2):
-//  * deep trees (p >= 128) with few columns -- at most 2048 16-byte column
-//    units, 4096 from p = 512 -- but more than 20 MB of inputs once
+//  * deep trees (p >= 128) with few columns -- at most 4096 16-byte column
+//    units, 8192 from p = 256 -- but more than 20 MB of inputs once
 //    p >= 1024: the hierarchical tile, one kernel with a walk of about
-//    p / 64 ranks per thread (p = 1152, m = 2^13, cold: 21.9 us against
-//    36.4 us for the tile and 38.5 us for the split layout);
+//    p / 64 (8 units per CTA) or p / 32 (16 units) ranks per thread
+//    (p = 1152, m = 2^13, cold: 22.2 us against 36.3 us for the tile and
+//    38.7 us for the split layout; m = 2^15: 63.1 against 68.4 us for the
+//    split layout);
 //  * deep trees whose p input rows total at most kTileMaxBytes: the
-//    shared-memory tile, the layout with the lowest fixed cost (p = 288,
-//    m = 2^15 int32: 22.6 us against the split layout's 27.3 us; at 75.5 MB,
-//    twice that, the split layout wins at p = 288, 576 and 1152);
+//    shared-memory tile, the layout with the lowest fixed cost (p = 192,
+//    m = 2^15 int32: 11.4 us against the split layout's 19.9 us and the
+//    hierarchical tile's 17.7 us; at 75.5 MB the split layout wins at
+//    p = 288, 576 and 1152);
 //  * deep trees (p >= kSplitMinRanks) above that: the split layout, whose
 //    read phase (first kernel) and write phase (second kernel) keep HBM
 //    traffic one-directional; at p = 1152 it beats column streaming up to
@@ -40,7 +66,7 @@ static bool tree_preferred(const Plan* P)
     if (P->p < 128) return false;
     const int64_t units = P->m * int64_t(P->esize) / 16;
     const int64_t bytes = int64_t(P->p) * P->m * P->esize;
-    if (units > (P->p >= 512 ? 4096 : 2048)) return false;
+    if (units > (P->p >= 256 ? 8192 : 4096)) return false;
     return P->p < 1024 || bytes > kTreeMinBytesLargeP;
 }
 
@@ -196,7 +222,8 @@ int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t m
     a.tree_r1 = P->tree_r1;
     a.tree_s = P->tree_s;
     a.tree_slots = P->tree_slots;
-    a.tree_tiles = (a.nvec + fused::kTreeUnits - 1) / fused::kTreeUnits;
+    a.tree_width = P->tree_width;
+    a.tree_tiles = P->tree_width ? (a.nvec + P->tree_width - 1) / P->tree_width : 0;
     if ((mode == 4 || mode == 5) && !vec) mode = 1;  // 16-byte rows only: stream instead
 
     switch (mode) {

@@ -208,13 +208,9 @@ struct Bulk {
         const size_t bar_off = size_t(kBulkStages + 2) * kBulkTile + slots;
         const size_t smem = bar_off + 2 * kBulkStages * sizeof(uint64_t);
         a.bulk_bar_off = int(bar_off);
-        if (int(smem) > P->smem_attr[3]) {
-            cudaError_t e = cudaFuncSetAttribute(fused_bulk_kernel<Op>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 int(smem));
-            if (e != cudaSuccess) return cuda_fail(e, "fused bulk attribute");
-            P->smem_attr[3] = int(smem);
-        }
+        if (int rc = grant_smem(reinterpret_cast<const void*>(&fused_bulk_kernel<Op>), smem,
+                                &P->smem_attr[3], "fused bulk attribute"))
+            return rc;
         int occ = 0;
         cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fused_bulk_kernel<Op>,
                                                                      kBulkThreads, smem);

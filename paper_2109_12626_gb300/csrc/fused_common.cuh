@@ -31,8 +31,10 @@ constexpr int kBulkConsumers = 256;                   // 8 warps
 constexpr int kBulkThreads = kBulkConsumers + 32;     // + producer warp
 constexpr int kBulkTile = kBulkConsumers * 16;        // bytes per rank row piece
 constexpr int kBulkStages = 16;
-constexpr int kTreeThreads = 512;                     // hierarchical tile: threads,
-constexpr int kTreeUnits = 8;                         // and 16-byte column units per CTA
+constexpr int kTreeThreads = 512;                     // hierarchical tile: threads per CTA,
+constexpr int kTreeUnitsNarrow = 8;                   // 16-byte column units per CTA below
+constexpr int kTreeUnitsWide = 16;                    // kTreeWideUnits units, and from there
+constexpr int64_t kTreeWideUnits = 4096;
 
 struct FusedArgs {
     const char* const* x;   // [p] rank inputs
@@ -66,7 +68,8 @@ struct FusedArgs {
     const int4* tree_lev;   // levels above the cut: (node, child_0, child_1) entries
     const int* tree_levoff; // [tree_nlev + 1]
     int tree_nseg, tree_nlev, tree_r0, tree_r1, tree_s, tree_slots;
-    int64_t tree_tiles;     // CTAs of kTreeUnits vector units
+    int64_t tree_tiles;     // CTAs of tree_width vector units
+    int tree_width;         // kTreeUnitsNarrow or kTreeUnitsWide
 };
 
 template <class Op>
@@ -181,6 +184,13 @@ __device__ __forceinline__ int one_slot_stride(int n)
 }
 
 // launchers, one per layout (dispatch on the plan's element type)
+// Raise kernel fn's dynamic shared memory limit on the current device to at
+// least `bytes`, never lowering it: the attribute belongs to the function and
+// is shared by every plan, so a plan that needs less must not take it away
+// from one that needs more.  *granted is the plan's cache of what it already
+// has (launches that fit skip the call).
+int grant_smem(const void* fn, size_t bytes, int* granted, const char* what);
+
 int launch_stream(Plan* P, FusedArgs a, cudaStream_t s);
 int launch_tile(Plan* P, FusedArgs a, cudaStream_t s);
 int launch_split(Plan* P, FusedArgs a, cudaStream_t s);

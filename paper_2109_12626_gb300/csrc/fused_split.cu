@@ -111,14 +111,13 @@ struct Split {
         const size_t smem = size_t(P->max_depth + 1) * kStreamThreads * sizeof(uint4);
         if (blocks > 0x7fffffff) return fail(DPDR_ERR_INVALID, "m too large");
         if (int(smem) > P->smem_attr[2]) {
-            cudaError_t e = cudaFuncSetAttribute(fused_split_reduce_kernel<Op>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 int(smem));
-            if (e == cudaSuccess)
-                e = cudaFuncSetAttribute(fused_split_finish_kernel<Op>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-            if (e != cudaSuccess) return cuda_fail(e, "fused split attribute");
-            P->smem_attr[2] = int(smem);
+            int granted = P->smem_attr[2];
+            if (int rc = grant_smem(reinterpret_cast<const void*>(&fused_split_reduce_kernel<Op>),
+                                    smem, &granted, "fused split attribute"))
+                return rc;
+            if (int rc = grant_smem(reinterpret_cast<const void*>(&fused_split_finish_kernel<Op>),
+                                    smem, &P->smem_attr[2], "fused split attribute"))
+                return rc;
         }
         const int groups = (P->p + a.group - 1) / a.group;
         fused_split_reduce_kernel<Op>

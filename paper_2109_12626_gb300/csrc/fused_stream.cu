@@ -31,13 +31,9 @@ struct Stream {
         const int64_t blocks = (units + kStreamThreads - 1) / kStreamThreads;
         const size_t smem = size_t(P->max_depth + 1) * kStreamThreads * sizeof(uint4);
         if (blocks > 0x7fffffff) return fail(DPDR_ERR_INVALID, "m too large");
-        if (int(smem) > P->smem_attr[0]) {
-            cudaError_t e = cudaFuncSetAttribute(fused_stream_kernel<Op>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 int(smem));
-            if (e != cudaSuccess) return cuda_fail(e, "fused stream attribute");
-            P->smem_attr[0] = int(smem);
-        }
+        if (int rc = grant_smem(reinterpret_cast<const void*>(&fused_stream_kernel<Op>), smem,
+                                &P->smem_attr[0], "fused stream attribute"))
+            return rc;
         fused_stream_kernel<Op><<<unsigned(blocks), kStreamThreads, smem, s>>>(a);
         return launched();
     }

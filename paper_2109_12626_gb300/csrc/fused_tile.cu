@@ -119,13 +119,9 @@ struct Tile {
         const int64_t scal_tiles = (a.nscalar + (int64_t(1) << lg_s) - 1) >> lg_s;
         const int64_t blocks = a.vec_tiles + scal_tiles;
         if (blocks > 0x7fffffff) return fail(DPDR_ERR_INVALID, "m too large");
-        if (int(smem) > P->smem_attr[1]) {
-            cudaError_t e = cudaFuncSetAttribute(fused_tile_kernel<Op>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 int(smem));
-            if (e != cudaSuccess) return cuda_fail(e, "fused tile attribute");
-            P->smem_attr[1] = int(smem);
-        }
+        if (int rc = grant_smem(reinterpret_cast<const void*>(&fused_tile_kernel<Op>), smem,
+                                &P->smem_attr[1], "fused tile attribute"))
+            return rc;
         fused_tile_kernel<Op><<<unsigned(blocks), kTileThreads, smem, s>>>(a);
         return launched();
     }

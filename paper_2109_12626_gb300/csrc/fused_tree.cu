@@ -1,5 +1,5 @@
 // fused_tree.cu -- hierarchical tile layout of the fused kernel: one CTA per
-// tile of kTreeUnits column units runs the whole fold of its columns.
+// tile of W column units (8 or 16) runs the whole fold of its columns.
 //
 //  1. The tree is cut at depth s (Sec. 1.1's trees are complete, so a
 //     depth-s node roots a contiguous post-order interval of ranks).  Each
@@ -54,15 +54,14 @@ __device__ __forceinline__ typename U::T walk_subtree(const FusedArgs& a, int lo
     return acc;
 }
 
-// The three phases for wu <= kTreeUnits units starting at u0 (16-byte units
-// with VecUnit, single elements with OneUnit); slot/stride are this
-// thread's walk slots.
-template <class U>
+// The three phases for wu <= W units starting at u0 (16-byte units with
+// VecUnit, single elements with OneUnit); slot/stride are this thread's
+// walk slots.
+template <class U, int W>
 __device__ __forceinline__ void tree_body(const FusedArgs& a, int64_t u0, int wu, uint4* smem,
                                           typename U::T* slot, int stride)
 {
     using T = typename U::T;
-    constexpr int W = kTreeUnits;
     const int tid = threadIdx.x;
     T* part = reinterpret_cast<T*>(smem + a.tree_slots * kTreeThreads);  // [nseg][W]
     T* yrow = part + a.tree_nseg * W;                                      // [W]
@@ -107,26 +106,28 @@ __device__ __forceinline__ void tree_body(const FusedArgs& a, int64_t u0, int wu
     }
 }
 
-template <class Op>
+// W column units per CTA: kTreeUnitsNarrow for few columns (more CTAs),
+// kTreeUnitsWide for more (longer rows per rank, half the CTAs).
+template <class Op, int W>
 __global__ void __launch_bounds__(kTreeThreads, 2)
 fused_tree_kernel(FusedArgs a)
 {
     extern __shared__ uint4 smem[];
     const int tid = threadIdx.x;
     if (blockIdx.x < a.tree_tiles) {
-        const int64_t u0 = int64_t(blockIdx.x) * kTreeUnits;
-        tree_body<VecUnit<Op>>(a, u0, int(lmin(kTreeUnits, a.nvec - u0)), smem, smem + tid,
-                               kTreeThreads);
+        const int64_t u0 = int64_t(blockIdx.x) * W;
+        tree_body<VecUnit<Op>, W>(a, u0, int(lmin(W, a.nvec - u0)), smem, smem + tid,
+                                  kTreeThreads);
     } else {  // ragged tail: the single elements after the 16-byte units
-        tree_body<OneUnit<Op>>(a, a.scalar_base, int(a.nscalar), smem, one_slots<Op>(smem, tid),
-                               one_slot_stride<Op>(kTreeThreads));
+        tree_body<OneUnit<Op>, W>(a, a.scalar_base, int(a.nscalar), smem,
+                                  one_slots<Op>(smem, tid), one_slot_stride<Op>(kTreeThreads));
     }
 }
 
 size_t tree_smem(const Plan* P)
 {
-    return (size_t(P->tree_slots) * kTreeThreads + size_t(P->tree_nseg) * kTreeUnits +
-            kTreeUnits) * sizeof(uint4);
+    return (size_t(P->tree_slots) * kTreeThreads + size_t(P->tree_nseg) * P->tree_width +
+            P->tree_width) * sizeof(uint4);
 }
 
 template <class Op>
@@ -136,14 +137,14 @@ struct Tree {
         const size_t smem = tree_smem(P);
         const int64_t blocks = a.tree_tiles + (a.nscalar ? 1 : 0);
         if (blocks > 0x7fffffff) return fail(DPDR_ERR_INVALID, "m too large");
-        if (int(smem) > P->smem_attr[4]) {
-            cudaError_t e = cudaFuncSetAttribute(fused_tree_kernel<Op>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 int(smem));
-            if (e != cudaSuccess) return cuda_fail(e, "fused tree attribute");
-            P->smem_attr[4] = int(smem);
-        }
-        fused_tree_kernel<Op><<<unsigned(blocks), kTreeThreads, smem, s>>>(a);
+        const bool wide = a.tree_width == kTreeUnitsWide;
+        const void* kern = wide ? reinterpret_cast<const void*>(&fused_tree_kernel<Op, kTreeUnitsWide>)
+                                : reinterpret_cast<const void*>(&fused_tree_kernel<Op, kTreeUnitsNarrow>);
+        if (int rc = grant_smem(kern, smem, &P->smem_attr[4], "fused tree attribute")) return rc;
+        if (wide)
+            fused_tree_kernel<Op, kTreeUnitsWide><<<unsigned(blocks), kTreeThreads, smem, s>>>(a);
+        else
+            fused_tree_kernel<Op, kTreeUnitsNarrow><<<unsigned(blocks), kTreeThreads, smem, s>>>(a);
         return launched();
     }
 };
@@ -154,8 +155,11 @@ int launch_tree(Plan* P, FusedArgs a, cudaStream_t s) { return dispatch<Tree>(P,
 
 }  // namespace fused
 
-// Tables of the hierarchical tile layout: the cut depth s (about
-// kTreeThreads / kTreeUnits subtrees, one walk per thread), the entries --
+// Tables of the hierarchical tile layout: the tile width W (kTreeUnitsWide
+// column units per CTA from kTreeWideUnits column units on: p = 1152,
+// m = 2^14, cold L2: 32 us against 42 us with 8; below that 8, which gives
+// twice the CTAs: m = 2^13: 22 against 25 us), the cut depth s (about
+// kTreeThreads / W subtrees, one walk per thread), the entries --
 // first the depth-s nodes with their subtree intervals, then the nodes above
 // the cut (lo = hi = the node) -- and, per level above the cut, deepest
 // first, (node, child_0, child_1) as entry indices.
@@ -164,8 +168,10 @@ int fused_tree_prepare(Plan* P)
     if (P->tree_ready) return DPDR_OK;
     const int p = P->p;
     const int trees = P->r0 >= 0 ? 2 : 1;
+    const int64_t units = P->m * int64_t(P->esize) / 16;
+    const int W = units >= fused::kTreeWideUnits ? fused::kTreeUnitsWide : fused::kTreeUnitsNarrow;
     int s = 0;
-    while (trees << s < fused::kTreeThreads / fused::kTreeUnits) s++;
+    while (trees << s < fused::kTreeThreads / W) s++;
     s = std::min(s, P->max_depth);
     std::vector<int> idx(p, -1);
     std::vector<int2> seg;
@@ -217,6 +223,7 @@ int fused_tree_prepare(Plan* P)
     P->tree_slots = P->max_depth - s + 1;
     P->tree_r0 = P->r0 >= 0 ? idx[P->r0] : -1;
     P->tree_r1 = idx[P->r1];
+    P->tree_width = W;
     P->tree_ready = true;
     return DPDR_OK;
 }

@@ -504,7 +504,7 @@ extern "C" int dpdr_plan_info(dpdr_plan_t h, int64_t* info, int n)
                                  P->d_ll_bytes + P->d_tree_bytes),
                          P->last_vector_path, P->split_s, P->split_nseg, P->split_group,
                          P->sched_slices_used, P->topo, P->last_host_path,
-                         schedule_transport(P)};
+                         schedule_transport(P), P->tree_ready ? P->tree_width : 0};
     const int k = int(sizeof v / sizeof v[0]);
     for (int i = 0; i < n; i++) info[i] = i < k ? v[i] : 0;
     return DPDR_OK;

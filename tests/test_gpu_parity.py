@@ -43,6 +43,9 @@ CASES = [
     # trees (depth 11), eight ranks per schedule CTA, a 131 KB tile row
     ("p8190_m33_int32", "int32", 10, 8190, 33, dict(lo=-1000, hi=1000), [1, 2]),
     ("p8190_m7_f32", "float32", 10, 8190, 7, dict(sigma=1.0), [1]),
+    # 4097 16-byte units per rank plus a ragged tail: the hierarchical tile
+    # takes its wide width (16 units per CTA) at a deep tree
+    ("p1152_m16390_f32", "float32", 11, 1152, 16390, dict(sigma=1.0), [2]),
 ]
 
 
@@ -178,6 +181,62 @@ def test_guard_words_untouched(pkg, orc, run):
     _check_all(ys, want)
     for bb in bases:
         assert bool((bb[m:] == 7.25).all())
+
+
+@pytest.mark.parametrize("p,m,width", [(1152, 16383, 8), (1152, 16384, 16), (32, 65541, 16),
+                                       (7, 70000, 16), (4094, 100, 8)])
+def test_tree_width(pkg, p, m, width):
+    """The hierarchical tile takes 16 column units per CTA from 4096 16-byte
+    units per rank on, 8 below."""
+    with pkg.Plan(p, m, "float32", 1) as plan:
+        plan.set(pkg.OPT_FUSED_MODE, 5)
+        assert plan.info()["tree_width"] == width
+
+
+AUTO = [  # p, m, kind, layout the automatic choice takes (1 stream, 2 tile,
+          # 3 split, 5 hierarchical tile)
+    (32, 1 << 27, "float32", 1), (36, 65536, "mat2x2u32", 1), (7, 1000, "int32", 2),
+    (1152, 4096, "int32", 2), (1152, 8192, "int32", 5), (1152, 32768, "int32", 5),
+    (1152, 32772, "int32", 3), (128, 16384, "float32", 5), (192, 32768, "int32", 2),
+    (288, 32768, "int32", 5), (288, 65536, "int32", 3), (4094, 2048, "int32", 5),
+    (1152, 1 << 22, "float32", 3)]
+
+
+@pytest.mark.parametrize("p,m,kind,mode", AUTO)
+def test_auto_layout_choice(pkg, p, m, kind, mode):
+    with pkg.Plan(p, m, kind, 1) as plan:
+        assert plan.info()["auto_mode"] == mode
+
+
+@pytest.mark.parametrize("mode", [2, 5], ids=["tile", "tree"])
+def test_interleaved_plans_keep_their_shared_memory(pkg, orc, mode):
+    """Plans of one element type whose fused kernels need different dynamic
+    shared memory, called alternately (larger, smaller, larger): the kernel's
+    limit belongs to the function, so the smaller plan must not take back
+    what the larger one was granted.  Tile rows of 3001 and 2001 ranks need
+    96 KB and 64 KB; the hierarchical tile at p = 4094 and 1152 needs 64 KB
+    and 56 KB (all above the 48 KB default)."""
+    kind, m = "int32", 1001
+    dev = torch.device("cuda:0")
+    sizes = (3000, 2000) if mode == 2 else (4094, 1152)
+    data = {}
+    plans = {}
+    try:
+        for p in sizes:
+            x = host_inputs(kind, 30 + p % 7, p, m, lo=-1000, hi=1000)
+            xs, _ = to_device(x, kind, dev)
+            data[p] = (xs, _want(orc, x, kind))
+            plans[p] = pkg.Plan(p, m, kind, 1)
+            plans[p].set(pkg.OPT_FUSED_MODE, mode)
+        for p in (sizes[0], sizes[1], sizes[0], sizes[1]):
+            xs, want = data[p]
+            ys, _ = empty_like_ranks(xs)
+            plans[p].allreduce(xs, ys)
+            plans[p].sync()
+            _check_all(ys, want)
+    finally:
+        for plan in plans.values():
+            plan.close()
 
 
 def test_m_zero_is_a_no_op(pkg):
