@@ -20,6 +20,21 @@ namespace dpdr {
 //   bits 3-7  depth d
 constexpr int kTapeKeep = 4;
 constexpr int kMaxDepth = 31;
+constexpr int kMaxSlices = 1024;   // column slices per rank of the schedule kernel
+
+// Dual-root exchange slot of one column slice of the schedule kernel: the
+// slice's share of the largest block, rounded up to 16 bytes, plus 48 bytes
+// for the rounding of slice bounds to 16-byte units and for the offset that
+// keeps every element congruent to the inputs modulo 16 bytes.  Each slice
+// has a slot of its own: slices run independently, and a slice's range
+// inside a block moves by a few elements from block to block, so slots
+// shared across slices would let a slice that is two blocks ahead overwrite
+// a neighbour's data before the dual root has read it.
+inline size_t ring_sub_bytes(int64_t maxblk, size_t esize, int slices)
+{
+    const int64_t share = (maxblk + slices - 1) / slices;
+    return (size_t(share) * esize + 15) / 16 * 16 + 48;
+}
 
 // Entries of the level table of the shared-memory tile fold: internal
 // nodes, deepest level first, as (node, child_1 or -1); child_0 = node-1.

@@ -258,12 +258,13 @@ static void free_plan(Plan* P)
     delete P;
 }
 
-// Size of one dual-root exchange slot: the largest block plus the offset
-// that keeps it congruent to the inputs modulo 16 bytes.
+// Bytes of one (root, parity) group of dual-root exchange slots: room for
+// the per-slice slots of any slice count up to kMaxSlices (see
+// ring_sub_bytes: slices x slot <= largest block + 79 bytes per slice).
 static size_t ring_slot(const Plan* P)
 {
-    const int64_t maxblk = (P->m + P->b - 1) / std::max(P->b, 1) + 4;
-    return align_up(size_t(maxblk) * P->esize + 16, 256);
+    const int64_t maxblk = (P->m + P->b - 1) / std::max(P->b, 1);
+    return align_up(size_t(maxblk) * P->esize + size_t(kMaxSlices) * 80, 256);
 }
 
 static int allocate(Plan* P)
@@ -447,7 +448,7 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
         P->sched_rpc = int(v);
         return schedule_configure(P);
     case DPDR_OPT_SCHED_SLICES:
-        if (v < 0 || v > 1024) return fail(DPDR_ERR_INVALID, "slices: 0..1024");
+        if (v < 0 || v > kMaxSlices) return fail(DPDR_ERR_INVALID, "slices: 0..1024");
         P->sched_slices = int(v);
         return schedule_configure(P);
     case DPDR_OPT_SPLIT_DEPTH: {

@@ -279,11 +279,12 @@ __device__ __forceinline__ void fold_children(const SchedArgs& a, char* dst, con
     if (t1) block_op<Op, kG>(a, dst, t1, dst, s, e);
 }
 
-__device__ __forceinline__ char* ring_base(const SchedArgs& a, int side, int j,
+__device__ __forceinline__ char* ring_base(const SchedArgs& a, int side, int j, int g,
                                            int64_t s, int epv, int es)
 {
-    char* slot = a.ring + (int64_t(side) * 2 + (j & 1)) * a.ring_slot;
-    return slot - (s - s % epv) * es;  // keeps element k congruent mod 16
+    // slot of (root side, block parity, slice g), ring_slot bytes each
+    char* slot = a.ring + ((int64_t(side) * 2 + (j & 1)) * a.nslices + g) * a.ring_slot;
+    return slot - (s - s % epv) * es;  // element k at slot + (k - s + s % epv) * es
 }
 
 // Round j of Algorithm 1 at rank i, column slice g.  The waits for the two
@@ -328,13 +329,13 @@ __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j, int 
     if (paired_root) {  // step 3 at a root: exchange partials with the dual
         if (!inb) return true;
         const int side = (i == a.r0) ? 0 : 1;
-        char* slot = ring_base(a, side, j, bs, Op::kEpv, Op::kEsize);
+        char* slot = ring_base(a, side, j, g, s, Op::kEpv, Op::kEsize);
         fold_children<Op, kG>(a, slot, t[0], t[1], xi, s, e);
         publish<kG>(a, up + i, uint32_t(j + 1), nullptr, 0, i);
         const int du = (i == a.r0) ? a.r1 : a.r0;
         const Wait wd{up + du, uint32_t(j + 1), 2};
         if (!cta_wait<kG>(a, &wd, 1, i, j)) return false;
-        const char* other = ring_base(a, 1 - side, j, bs, Op::kEpv, Op::kEsize);
+        const char* other = ring_base(a, 1 - side, j, g, s, Op::kEpv, Op::kEsize);
         if (i == a.r0)  // lower root: Y[j] (.) t
             block_op<Op, kG>(a, yi, slot, other, s, e);
         else  // higher root: t (.) Y[j]
@@ -531,7 +532,9 @@ int schedule_launch(Plan* P, cudaStream_t s)
     a.abort_flag = P->d_ctrl + 2 * cw;
     a.err = P->d_err;
     a.ring = P->d_ring;
-    a.ring_slot = int64_t(P->ring_slot_bytes);
+    a.ring_slot = int64_t(ring_sub_bytes((P->m + P->b - 1) / P->b, P->esize, P->sched_slices_used));
+    if (size_t(a.ring_slot) * P->sched_slices_used > P->ring_slot_bytes)
+        return fail(DPDR_ERR_INVALID, "schedule: exchange slots too small for the slice count");
     a.p = P->p;
     a.b = P->b;
     a.r0 = P->r0;
@@ -596,8 +599,7 @@ inline NoAllocLayout noalloc_layout(int p, int64_t m, int b, size_t esize)
     L.err = na_align(L.ctrl + sizeof(uint32_t) * (2 * size_t(p) + 1));
     L.cta = na_align(L.err + sizeof(uint32_t) * 4);
     L.ring = na_align(L.cta + sizeof(int) * (size_t(p) + 2));
-    const int64_t maxblk = (m + b - 1) / b + 4;
-    L.slot = na_align(size_t(maxblk) * esize + 16);
+    L.slot = na_align(ring_sub_bytes((m + b - 1) / b, esize, 1));
     L.end = L.ring + 4 * L.slot;
     return L;
 }

@@ -512,6 +512,38 @@ def test_int32_sums_wrap(pkg, orc, run):
     _check_all(ys, want)
 
 
+@pytest.mark.parametrize("kind,p,m,b", [("int32", 288, 2500000, 86), ("float32", 32, 2500000, 86),
+                                        ("mat2x2u32", 36, 300001, 7)])
+def test_schedule_slices_with_shifting_block_bounds(pkg, orc, kind, p, m, b):
+    """Blocks of two lengths (m mod b of them one element longer) cut into
+    column slices, with the counters transport: a slice's range inside a
+    block moves by a few elements from block to block and slices run
+    independently, so each slice has its own dual-root exchange slots (with
+    slots shared across slices, a slice two blocks ahead overwrote its
+    neighbour's data before the other root had read it)."""
+    rng = np.random.default_rng(90 + p)
+    if kind == "int32":
+        x = rng.integers(-1000, 1000, (p, m), dtype=np.int32)
+    elif kind == "float32":
+        x = rng.standard_normal((p, m)).astype(np.float32)
+    else:
+        x = rng.integers(0, 1 << 32, (p, m, 4), dtype=np.uint32)
+    want = _want(orc, x, kind).reshape(1, -1)
+    dev = torch.device("cuda:0")
+    xt = torch.from_numpy(x.view(np.int32)).to(dev)
+    xs = list(xt.unbind(0))
+    with pkg.Plan(p, m, kind, b) as plan:
+        plan.set(pkg.OPT_SCHED_TRANSPORT, 1)
+        assert plan.info()["sched_slices"] > 1
+        for _ in range(3):  # the overwrite was a race: several runs
+            yt = torch.full_like(xt, -3)
+            plan.allreduce_schedule(xs, list(yt.unbind(0)))
+            plan.sync()
+            got = yt.cpu().numpy().reshape(p, -1)
+            bad = np.nonzero((got != want).any(axis=1))[0]
+            assert bad.size == 0, "%d ranks differ, first %d" % (bad.size, bad[0])
+
+
 @pytest.mark.parametrize("run", ["fused_auto", "fused_stream", "fused_tree", "fused_split",
                                  "schedule_auto"])
 def test_very_many_ranks(pkg, orc, run):
