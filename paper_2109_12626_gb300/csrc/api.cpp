@@ -229,7 +229,8 @@ extern "C" int dpdr_allreduce_host(dpdr_plan_t h, const void* const* x_host,
     if (P->m == 0) return DPDR_OK;
     // direct: one launch loads the inputs from host memory and stores the
     // result to host memory, the link carrying both directions at once.  The
-    // layout DPDR_OPT_FUSED_MODE names, else the hierarchical tile, whose
+    // layout DPDR_OPT_FUSED_MODE names, else the hierarchical tile (8 column
+    // units per CTA at every size, whose extra CTAs help here), whose
     // CTAs read all their columns, then write them, and drift out of phase
     // with each other (p = 1152, m = 2^20: 297 GB/s against 230 for column
     // streaming, whose threads read and write in long lockstep phases at
@@ -248,7 +249,7 @@ extern "C" int dpdr_allreduce_host(dpdr_plan_t h, const void* const* x_host,
         const int mode = P->fused_mode ? P->fused_mode : stream ? 1 : 5;
         if (mode == 5 && (rc = fused_tree_prepare(P)) != DPDR_OK) return rc;
         P->last_host_path = 2;
-        return fused_launch_cols(P, P->d_x, P->d_y, P->m, P->last_vector_path != 0, s, mode);
+        return fused_launch_cols(P, P->d_x, P->d_y, P->m, P->last_vector_path != 0, s, mode, 0);
     }
     if (P->host_path == 2)
         return fail(DPDR_ERR_INVALID, "dpdr_allreduce_host: host buffers not addressable by the GPU");

@@ -43,6 +43,20 @@ struct LevelNode {
     int child1;
 };
 
+// Tables of the hierarchical tile layout for one tile width (fused_tree.cu):
+// the entries (subtrees at depth s, then the nodes above the cut) and the
+// level table above the cut.
+struct TreeTables {
+    bool ready = false;
+    int width = 0;                   // 16-byte column units per CTA
+    int s = 0, nseg = 0, nlev = 0, slots = 0, r0 = -1, r1 = 0;
+    char* d = nullptr;               // own allocation
+    size_t bytes = 0;
+    int2* seg = nullptr;
+    int4* lev = nullptr;
+    int* levoff = nullptr;
+};
+
 struct Plan {
     int p = 0;
     int64_t m = 0;
@@ -104,9 +118,10 @@ struct Plan {
     bool staged_pending = false;     // d_x / d_y hold last_x / last_y
 
     // dynamic shared memory already granted to the fused kernels of this
-    // plan's element type (stream, tile, split, bulk, hierarchical tile), so
+    // plan's element type (stream, tile, split, bulk, hierarchical tile of
+    // either width), so
     // launches skip the attribute call; the limits themselves only ever rise
-    int smem_attr[5] = {48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024};
+    int smem_attr[6] = {48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024};
 
     // split layout of the fused kernel (fused.cu): subtrees at depth split_s
     bool split_ready = false;
@@ -118,16 +133,9 @@ struct Plan {
     char* d_part = nullptr;
     int64_t part_stride = 0;
 
-    // hierarchical tile layout of the fused kernel (fused_tree.cu): entries
-    // (subtrees at depth tree_s, then nodes above the cut) and level table
-    bool tree_ready = false;
-    int tree_s = 0, tree_nseg = 0, tree_nlev = 0, tree_slots = 0, tree_r0 = -1, tree_r1 = 0;
-    int tree_width = 0;              // column units per CTA
-    char* d_tree = nullptr;          // own allocation
-    size_t d_tree_bytes = 0;
-    int2* d_tree_seg = nullptr;
-    int4* d_tree_lev = nullptr;
-    int* d_tree_levoff = nullptr;
+    // hierarchical tile layout of the fused kernel (fused_tree.cu), one set
+    // of tables per tile width: [0] 8 column units per CTA, [1] 16
+    TreeTables tree[2];
 
     // host-buffer pipeline of dpdr_allreduce_host (api.cpp), made on first use:
     // column chunks copied in on one stream, reduced on the caller's stream,
@@ -169,10 +177,12 @@ int stage_pointers(Plan* P, const void* const* x, const void* const* y,
 // launchers
 int fused_launch(Plan* P, cudaStream_t s);      // fused.cu
 int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t mc, bool vec,
-                      cudaStream_t s, int force_mode);  // fused.cu (0: plan's choice)
+                      cudaStream_t s, int force_mode,  // fused.cu (0: plan's choice)
+                      int tree_index = -1);  // hierarchical tile width: -1 plan's, 0 / 1
 int fused_auto_mode(const Plan* P);             // fused.cu
 int fused_split_prepare(Plan* P, bool force, int depth);  // fused.cu
-int fused_tree_prepare(Plan* P);                // fused_tree.cu
+int fused_tree_prepare(Plan* P);                // fused_tree.cu: both widths
+int fused_tree_index(const Plan* P);            // fused_tree.cu: the device path's width
 int schedule_launch(Plan* P, cudaStream_t s);   // schedule.cu
 int schedule_configure(Plan* P);                // schedule.cu
 int schedule_plan_rpc(Plan* P);                 // schedule.cu: ranks per CTA only

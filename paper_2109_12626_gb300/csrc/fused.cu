@@ -79,7 +79,7 @@ static bool tile_preferred(const Plan* P)
 int fused_auto_mode(const Plan* P)
 {
     const int64_t units = P->m * int64_t(P->esize) / 16;
-    if (P->tree_ready && tree_preferred(P)) return 5;
+    if (P->tree[fused_tree_index(P)].ready && tree_preferred(P)) return 5;
     if (tile_preferred(P)) return 2;
     if (P->p >= kSplitMinRanks && units >= 4096 && P->split_ready) return 3;
     if (units >= stream_target(P) / 4) return 1;
@@ -176,14 +176,15 @@ int fused_launch(Plan* P, cudaStream_t s)
 // The fused kernel on mc columns, with device tables of rank pointers that
 // may point into the middle of the rank buffers (a column chunk).
 int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t mc, bool vec,
-                      cudaStream_t s, int force_mode)
+                      cudaStream_t s, int force_mode, int tree_index)
 {
     if (mc == 0) return DPDR_OK;
     int mode = force_mode ? force_mode : P->fused_mode ? P->fused_mode : fused_auto_mode(P);
     const int lg = tile_lg_wu(P);
     if (mode == 2 && lg < 0) return fail(DPDR_ERR_INVALID, "tile mode: p too large");
     if (mode == 3 && !P->split_ready) return fail(DPDR_ERR_INVALID, "split mode: p < 2");
-    if (mode == 5 && !P->tree_ready) return fail(DPDR_ERR_INVALID, "tree mode not prepared");
+    const TreeTables& T = P->tree[tree_index < 0 ? fused_tree_index(P) : tree_index];
+    if (mode == 5 && !T.ready) return fail(DPDR_ERR_INVALID, "tree mode not prepared");
     if (mode < 1 || mode > 5) return fail(DPDR_ERR_INVALID, "unknown fused mode");
 
     FusedArgs a;
@@ -213,17 +214,17 @@ int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t m
     a.bulk_bar_off = 0;
     a.err = P->d_err;
     a.wait_ns = P->wait_ns;
-    a.tree_seg = P->d_tree_seg;
-    a.tree_lev = P->d_tree_lev;
-    a.tree_levoff = P->d_tree_levoff;
-    a.tree_nseg = P->tree_nseg;
-    a.tree_nlev = P->tree_nlev;
-    a.tree_r0 = P->tree_r0;
-    a.tree_r1 = P->tree_r1;
-    a.tree_s = P->tree_s;
-    a.tree_slots = P->tree_slots;
-    a.tree_width = P->tree_width;
-    a.tree_tiles = P->tree_width ? (a.nvec + P->tree_width - 1) / P->tree_width : 0;
+    a.tree_seg = T.seg;
+    a.tree_lev = T.lev;
+    a.tree_levoff = T.levoff;
+    a.tree_nseg = T.nseg;
+    a.tree_nlev = T.nlev;
+    a.tree_r0 = T.r0;
+    a.tree_r1 = T.r1;
+    a.tree_s = T.s;
+    a.tree_slots = T.slots;
+    a.tree_width = T.width;
+    a.tree_tiles = T.width ? (a.nvec + T.width - 1) / T.width : 0;
     if ((mode == 4 || mode == 5) && !vec) mode = 1;  // 16-byte rows only: stream instead
 
     switch (mode) {

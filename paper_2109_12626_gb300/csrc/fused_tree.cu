@@ -124,23 +124,24 @@ fused_tree_kernel(FusedArgs a)
     }
 }
 
-size_t tree_smem(const Plan* P)
+size_t tree_smem(const FusedArgs& a)
 {
-    return (size_t(P->tree_slots) * kTreeThreads + size_t(P->tree_nseg) * P->tree_width +
-            P->tree_width) * sizeof(uint4);
+    return (size_t(a.tree_slots) * kTreeThreads + size_t(a.tree_nseg) * a.tree_width +
+            a.tree_width) * sizeof(uint4);
 }
 
 template <class Op>
 struct Tree {
     static int run(Plan* P, FusedArgs a, cudaStream_t s)
     {
-        const size_t smem = tree_smem(P);
+        const size_t smem = tree_smem(a);
         const int64_t blocks = a.tree_tiles + (a.nscalar ? 1 : 0);
         if (blocks > 0x7fffffff) return fail(DPDR_ERR_INVALID, "m too large");
         const bool wide = a.tree_width == kTreeUnitsWide;
         const void* kern = wide ? reinterpret_cast<const void*>(&fused_tree_kernel<Op, kTreeUnitsWide>)
                                 : reinterpret_cast<const void*>(&fused_tree_kernel<Op, kTreeUnitsNarrow>);
-        if (int rc = grant_smem(kern, smem, &P->smem_attr[4], "fused tree attribute")) return rc;
+        if (int rc = grant_smem(kern, smem, &P->smem_attr[wide ? 5 : 4], "fused tree attribute"))
+            return rc;
         if (wide)
             fused_tree_kernel<Op, kTreeUnitsWide><<<unsigned(blocks), kTreeThreads, smem, s>>>(a);
         else
@@ -155,21 +156,27 @@ int launch_tree(Plan* P, FusedArgs a, cudaStream_t s) { return dispatch<Tree>(P,
 
 }  // namespace fused
 
-// Tables of the hierarchical tile layout: the tile width W (kTreeUnitsWide
-// column units per CTA from kTreeWideUnits column units on: p = 1152,
-// m = 2^14, cold L2: 32 us against 42 us with 8; below that 8, which gives
-// twice the CTAs: m = 2^13: 22 against 25 us), the cut depth s (about
-// kTreeThreads / W subtrees, one walk per thread), the entries --
+// The tile width of the device path: kTreeUnitsWide column units per CTA
+// from kTreeWideUnits column units per rank on (p = 1152, m = 2^14, cold L2:
+// 32 us against 42 us with 8), else kTreeUnitsNarrow, which gives twice the
+// CTAs (m = 2^13: 22 against 25 us).  The host-buffer path always takes the
+// narrow tile: over the host link, more CTAs drifting out of phase keep both
+// directions busier (p = 1152, m = 2^20: 297 against 272 GB/s).
+int fused_tree_index(const Plan* P)
+{
+    return P->m * int64_t(P->esize) / 16 >= fused::kTreeWideUnits ? 1 : 0;
+}
+
+// Tables of the hierarchical tile layout for tile width W: the cut depth s
+// (about kTreeThreads / W subtrees, one walk per thread), the entries --
 // first the depth-s nodes with their subtree intervals, then the nodes above
 // the cut (lo = hi = the node) -- and, per level above the cut, deepest
 // first, (node, child_0, child_1) as entry indices.
-int fused_tree_prepare(Plan* P)
+static int tree_tables(Plan* P, int W, TreeTables* T)
 {
-    if (P->tree_ready) return DPDR_OK;
+    if (T->ready) return DPDR_OK;
     const int p = P->p;
     const int trees = P->r0 >= 0 ? 2 : 1;
-    const int64_t units = P->m * int64_t(P->esize) / 16;
-    const int W = units >= fused::kTreeWideUnits ? fused::kTreeUnitsWide : fused::kTreeUnitsNarrow;
     int s = 0;
     while (trees << s < fused::kTreeThreads / W) s++;
     s = std::min(s, P->max_depth);
@@ -212,20 +219,26 @@ int fused_tree_prepare(Plan* P)
         cudaFree(d);
         return cuda_fail(e, "tree layout: upload");
     }
-    P->d_tree = d;
-    P->d_tree_bytes = bytes;
-    P->d_tree_seg = reinterpret_cast<int2*>(d);
-    P->d_tree_lev = reinterpret_cast<int4*>(d + o_lev);
-    P->d_tree_levoff = reinterpret_cast<int*>(d + o_off);
-    P->tree_s = s;
-    P->tree_nseg = int(seg.size());
-    P->tree_nlev = int(off.size()) - 1;
-    P->tree_slots = P->max_depth - s + 1;
-    P->tree_r0 = P->r0 >= 0 ? idx[P->r0] : -1;
-    P->tree_r1 = idx[P->r1];
-    P->tree_width = W;
-    P->tree_ready = true;
+    T->d = d;
+    T->bytes = bytes;
+    T->seg = reinterpret_cast<int2*>(d);
+    T->lev = reinterpret_cast<int4*>(d + o_lev);
+    T->levoff = reinterpret_cast<int*>(d + o_off);
+    T->s = s;
+    T->nseg = int(seg.size());
+    T->nlev = int(off.size()) - 1;
+    T->slots = P->max_depth - s + 1;
+    T->r0 = P->r0 >= 0 ? idx[P->r0] : -1;
+    T->r1 = idx[P->r1];
+    T->width = W;
+    T->ready = true;
     return DPDR_OK;
+}
+
+int fused_tree_prepare(Plan* P)
+{
+    int rc = tree_tables(P, fused::kTreeUnitsNarrow, &P->tree[0]);
+    return rc ? rc : tree_tables(P, fused::kTreeUnitsWide, &P->tree[1]);
 }
 
 }  // namespace dpdr

@@ -250,7 +250,8 @@ static void free_plan(Plan* P)
     if (P->pipe_out) cudaStreamDestroy(P->pipe_out);
     if (P->d_pipe) cudaFree(P->d_pipe);
     if (P->d_split) cudaFree(P->d_split);
-    if (P->d_tree) cudaFree(P->d_tree);
+    for (TreeTables& T : P->tree)
+        if (T.d) cudaFree(T.d);
     if (P->d_sched) cudaFree(P->d_sched);
     if (P->d_ll) cudaFree(P->d_ll);
     if (P->h_ptrs) cudaFreeHost(P->h_ptrs);
@@ -502,10 +503,10 @@ extern "C" int dpdr_plan_info(dpdr_plan_t h, int64_t* info, int n)
     const int64_t v[] = {P->p, P->m, P->b, P->max_depth, fused_auto_mode(P),
                          P->sched_ctas, P->sched_ranks_per_cta,
                          int64_t(P->dmem_bytes + P->d_split_bytes + P->d_sched_bytes +
-                                 P->d_ll_bytes + P->d_tree_bytes),
+                                 P->d_ll_bytes + P->tree[0].bytes + P->tree[1].bytes),
                          P->last_vector_path, P->split_s, P->split_nseg, P->split_group,
                          P->sched_slices_used, P->topo, P->last_host_path,
-                         schedule_transport(P), P->tree_ready ? P->tree_width : 0};
+                         schedule_transport(P), P->tree[fused_tree_index(P)].width};
     const int k = int(sizeof v / sizeof v[0]);
     for (int i = 0; i < n; i++) info[i] = i < k ? v[i] : 0;
     return DPDR_OK;

@@ -272,7 +272,9 @@ def test_repeated_calls_and_pointer_changes(pkg, orc):
 
 @pytest.mark.parametrize("kind,p,m,chunk", [("float32", 32, 10007, 0), ("float32", 32, 10007, 4096),
                                             ("int32", 1152, 3001, 65536), ("mat2x2u32", 7, 2049, 4096),
-                                            ("float32", 3, 257, 4096), ("mat2x2f32", 36, 1001, 0)])
+                                            ("float32", 3, 257, 4096), ("mat2x2f32", 36, 1001, 0),
+                                            # device buffers: 16 units per CTA; host: 8
+                                            ("float32", 300, 16390, 0)])
 @pytest.mark.parametrize("path", ["auto", "copy"])
 @pytest.mark.parametrize("pinned", [True, False])
 @pytest.mark.parametrize("in_place", [False, True])
