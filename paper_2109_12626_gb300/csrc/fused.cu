@@ -1,6 +1,7 @@
 // fused.cu -- layout choice and launch of the fused bandwidth kernel
 // (dpdr_allreduce); the layouts themselves live in fused_stream.cu,
 // fused_tile.cu, fused_split.cu and fused_bulk.cu (see fused_common.cuh).
+#include <algorithm>
 #include <map>
 #include <mutex>
 #include <utility>
@@ -36,14 +37,20 @@ using fused::tile_lg_wu;
 static int64_t stream_target(const Plan* P) { return int64_t(P->num_sms) * 1024; }
 
 // Layout choice, from layout sweeps measured on GB300 (int32, p = 128 ...
-// 4096, m = 2^10 ... 2^20, warm and cold L2):
+// 4096, m = 2^10 ... 2^20, warm and cold L2; where the two disagree, cold
+// decides unless warm is far ahead):
 //  * deep trees (p >= 128) with few columns -- at most 4096 16-byte column
 //    units, 8192 from p = 256 -- but more than 20 MB of inputs once
 //    p >= 1024: the hierarchical tile, one kernel with a walk of about
 //    p / 64 (8 units per CTA) or p / 32 (16 units) ranks per thread
-//    (p = 1152, m = 2^13, cold: 22.2 us against 36.3 us for the tile and
-//    38.7 us for the split layout; m = 2^15: 63.1 against 68.4 us for the
-//    split layout);
+//    (p = 1152, m = 2^13, cold: 22.2 us against 36.2 us for the tile and
+//    38.5 us for the split layout; m = 2^15: 63.6 against 67.1 us for the
+//    split layout).  Both tiles take their time in waves of resident CTAs,
+//    so where the shared-memory tile needs fewer waves than the
+//    hierarchical one, the shared-memory tile takes over (p = 288,
+//    m = 24576: one wave against two, 13.2 us warm and 18.3 cold against
+//    19.3 and 21.7; with as many waves the hierarchical tile is ahead or
+//    level: p = 256, m = 2^15, 17.5/20.8 against 19.8/26.3);
 //  * deep trees whose p input rows total at most kTileMaxBytes: the
 //    shared-memory tile, the layout with the lowest fixed cost (p = 192,
 //    m = 2^15 int32: 11.4 us against the split layout's 19.9 us and the
@@ -61,6 +68,15 @@ constexpr int kSplitMinRanks = 128;
 constexpr int64_t kSplitWork = int64_t(1) << 17;
 constexpr int64_t kTreeMinBytesLargeP = int64_t(20) << 20;
 
+// Resident CTAs of the shared-memory tile on the GPU: up to 4 per SM (256
+// threads of 64 registers), fewer when its rows do not fit the 228 KB of
+// shared memory per SM (1 KB of which is reserved per CTA).
+static int64_t tile_slots(const Plan* P)
+{
+    const size_t smem = size_t(P->p + 1) * (size_t(16) << tile_lg_wu(P));
+    return int64_t(P->num_sms) * std::min<int64_t>(4, int64_t((228 << 10) / (smem + 1024)));
+}
+
 static bool tree_preferred(const Plan* P)
 {
     if (P->p < 128) return false;
@@ -68,6 +84,21 @@ static bool tree_preferred(const Plan* P)
     const int64_t bytes = int64_t(P->p) * P->m * P->esize;
     if (units > (P->p >= 256 ? 8192 : 4096)) return false;
     return P->p < 1024 || bytes > kTreeMinBytesLargeP;
+}
+
+// Whether the shared-memory tile needs fewer waves of resident CTAs than
+// the hierarchical tile for the plan's columns.
+static bool tile_beats_tree(const Plan* P)
+{
+    const int lg = tile_lg_wu(P);
+    if (lg < 0) return false;
+    const int64_t units = P->m * int64_t(P->esize) / 16;
+    const int64_t W = P->tree[fused_tree_index(P)].width;
+    const int64_t tree_slots = int64_t(fused::kTreeCtasPerSm) * P->num_sms;
+    const int64_t tiles = (units + (int64_t(1) << lg) - 1) >> lg;
+    const int64_t tree_waves = ((units + W - 1) / W + tree_slots - 1) / tree_slots;
+    const int64_t tile_waves = (tiles + tile_slots(P) - 1) / tile_slots(P);
+    return tile_waves < tree_waves;
 }
 
 static bool tile_preferred(const Plan* P)
@@ -79,7 +110,8 @@ static bool tile_preferred(const Plan* P)
 int fused_auto_mode(const Plan* P)
 {
     const int64_t units = P->m * int64_t(P->esize) / 16;
-    if (P->tree[fused_tree_index(P)].ready && tree_preferred(P)) return 5;
+    if (P->tree[fused_tree_index(P)].ready && tree_preferred(P))
+        return tile_beats_tree(P) ? 2 : 5;
     if (tile_preferred(P)) return 2;
     if (P->p >= kSplitMinRanks && units >= 4096 && P->split_ready) return 3;
     if (units >= stream_target(P) / 4) return 1;

@@ -32,9 +32,9 @@ constexpr int kBulkThreads = kBulkConsumers + 32;     // + producer warp
 constexpr int kBulkTile = kBulkConsumers * 16;        // bytes per rank row piece
 constexpr int kBulkStages = 16;
 constexpr int kTreeThreads = 512;                     // hierarchical tile: threads per CTA,
-constexpr int kTreeUnitsNarrow = 8;                   // 16-byte column units per CTA below
-constexpr int kTreeUnitsWide = 16;                    // kTreeWideUnits units, and from there
-constexpr int64_t kTreeWideUnits = 4096;
+constexpr int kTreeUnitsNarrow = 8;                   // 16-byte column units per CTA:
+constexpr int kTreeUnitsWide = 16;                    // the two tile widths
+constexpr int kTreeCtasPerSm = 2;                     // resident (registers, shared memory)
 
 struct FusedArgs {
     const char* const* x;   // [p] rank inputs

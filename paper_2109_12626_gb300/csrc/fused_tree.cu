@@ -156,15 +156,20 @@ int launch_tree(Plan* P, FusedArgs a, cudaStream_t s) { return dispatch<Tree>(P,
 
 }  // namespace fused
 
-// The tile width of the device path: kTreeUnitsWide column units per CTA
-// from kTreeWideUnits column units per rank on (p = 1152, m = 2^14, cold L2:
-// 32 us against 42 us with 8), else kTreeUnitsNarrow, which gives twice the
-// CTAs (m = 2^13: 22 against 25 us).  The host-buffer path always takes the
-// narrow tile: over the host link, more CTAs drifting out of phase keep both
-// directions busier (p = 1152, m = 2^20: 297 against 272 GB/s).
+// The tile width of the device path: kTreeUnitsNarrow column units per CTA
+// while those CTAs fit in one wave of resident CTAs, else kTreeUnitsWide,
+// whose CTAs cost about 1.6 times as much but are half as many (p = 1152,
+// int32, cold L2: m = 2^13, one narrow wave: 22.2 against 24.6 us; m = 10240,
+// two narrow waves against one wide: 38.8 against 28.9 us; m = 2^15, four
+// against two: 81.5 against 63.6 us; from p = 256 to 2304 alike).  The
+// host-buffer path always takes the narrow tile: over the host link, more
+// CTAs drifting out of phase keep both directions busier (p = 1152,
+// m = 2^20: 297 against 272 GB/s).
 int fused_tree_index(const Plan* P)
 {
-    return P->m * int64_t(P->esize) / 16 >= fused::kTreeWideUnits ? 1 : 0;
+    const int64_t units = P->m * int64_t(P->esize) / 16;
+    const int64_t slots = int64_t(fused::kTreeCtasPerSm) * P->num_sms;
+    return units > fused::kTreeUnitsNarrow * slots ? 1 : 0;
 }
 
 // Tables of the hierarchical tile layout for tile width W: the cut depth s

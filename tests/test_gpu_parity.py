@@ -183,29 +183,37 @@ def test_guard_words_untouched(pkg, orc, run):
         assert bool((bb[m:] == 7.25).all())
 
 
-@pytest.mark.parametrize("p,m,width", [(1152, 16383, 8), (1152, 16384, 16), (32, 65541, 16),
-                                       (7, 70000, 16), (4094, 100, 8)])
-def test_tree_width(pkg, p, m, width):
-    """The hierarchical tile takes 16 column units per CTA from 4096 16-byte
-    units per rank on, 8 below."""
-    with pkg.Plan(p, m, "float32", 1) as plan:
-        plan.set(pkg.OPT_FUSED_MODE, 5)
-        assert plan.info()["tree_width"] == width
-
-
-AUTO = [  # p, m, kind, layout the automatic choice takes (1 stream, 2 tile,
-          # 3 split, 5 hierarchical tile)
+AUTO = [  # p, m, kind, layout the automatic choice takes on a 152-SM GPU
+          # (1 stream, 2 tile, 3 split, 5 hierarchical tile)
     (32, 1 << 27, "float32", 1), (36, 65536, "mat2x2u32", 1), (7, 1000, "int32", 2),
     (1152, 4096, "int32", 2), (1152, 8192, "int32", 5), (1152, 32768, "int32", 5),
     (1152, 32772, "int32", 3), (128, 16384, "float32", 5), (192, 32768, "int32", 2),
     (288, 32768, "int32", 5), (288, 65536, "int32", 3), (4094, 2048, "int32", 5),
-    (1152, 1 << 22, "float32", 3)]
+    (1152, 1 << 22, "float32", 3),
+    # the shared-memory tile where it needs fewer waves of resident CTAs
+    # than the hierarchical tile (p = 288: one against two)
+    (288, 24576, "int32", 2), (288, 16384, "int32", 5), (576, 24576, "int32", 5),
+    (576, 32768, "int32", 5), (768, 24576, "int32", 5), (256, 28672, "int32", 2)]
 
 
 @pytest.mark.parametrize("p,m,kind,mode", AUTO)
 def test_auto_layout_choice(pkg, p, m, kind, mode):
+    if torch.cuda.get_device_properties(0).multi_processor_count != 152:
+        pytest.skip("the expected choices are for a 152-SM GPU")
     with pkg.Plan(p, m, kind, 1) as plan:
         assert plan.info()["auto_mode"] == mode
+
+
+@pytest.mark.parametrize("p,m", [(1152, 9728), (1152, 9732), (1152, 16384), (32, 65541),
+                                 (7, 70000), (4094, 100), (300, 40000)])
+def test_tree_width(pkg, p, m):
+    """On device buffers the hierarchical tile takes 8 column units per CTA
+    while those CTAs fit in one wave of resident CTAs (2 per SM), else 16."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    units = m * 4 // 16
+    with pkg.Plan(p, m, "float32", 1) as plan:
+        plan.set(pkg.OPT_FUSED_MODE, 5)
+        assert plan.info()["tree_width"] == (16 if units > 8 * 2 * sms else 8)
 
 
 @pytest.mark.parametrize("mode", [2, 5], ids=["tile", "tree"])
