@@ -215,8 +215,8 @@ int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
  *   [14] path of the last dpdr_allreduce_host: 1 copy pipeline, 2 direct
  *   [15] transport of dpdr_allreduce_schedule: 1 counters, 2 flagged words
  *   [16] 16-byte column units per CTA of the hierarchical tile layout on
- *        device buffers (8, or 16 from 4096 units per rank; host buffers
- *        always take 8) */
+ *        device buffers (8 while those CTAs fit in one wave of resident
+ *        CTAs, 2 per SM; else 16; host buffers always take 8) */
 int dpdr_plan_info(dpdr_plan_t plan, int64_t* info, int n);
 
 /* Releases the plan's device and host memory.  The caller must first make
