@@ -9,7 +9,7 @@ The draws reach combinations no hand-written case names -- blocks of two
 lengths cut into slices, ragged tails under every layout, deep trees with
 few columns -- and a mismatch names its case number, which reproduces it.
 DPDR_FUZZ_CASES and DPDR_FUZZ_LARGE_CASES set the number of cases (default
-128 up to 16 MB of inputs and 16 up to 256 MB)."""
+128 up to 16 MB of inputs and 32 up to 256 MB)."""
 import os
 
 import numpy as np
@@ -107,7 +107,7 @@ def test_random_configuration(pkg, orc, k):
                     assert np.array_equal(bits(xs[i]), expect_bits(x[i])), (k, run, i)
 
 
-N_LARGE = int(os.environ.get("DPDR_FUZZ_LARGE_CASES", "16"))
+N_LARGE = int(os.environ.get("DPDR_FUZZ_LARGE_CASES", "32"))
 
 
 def draw_large(k: int) -> dict:
