@@ -119,9 +119,10 @@ struct Plan {
 
     // dynamic shared memory already granted to the fused kernels of this
     // plan's element type (stream, tile, split, bulk, hierarchical tile of
-    // either width), so
+    // either width, paired stream), so
     // launches skip the attribute call; the limits themselves only ever rise
-    int smem_attr[6] = {48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024};
+    int smem_attr[7] = {48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024, 48 * 1024,
+                        48 * 1024};
 
     // split layout of the fused kernel (fused.cu): subtrees at depth split_s
     bool split_ready = false;
