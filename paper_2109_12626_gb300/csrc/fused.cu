@@ -60,9 +60,11 @@ static int64_t stream_target(const Plan* P) { return int64_t(P->num_sms) * 1024;
 //    read phase (first kernel) and write phase (second kernel) keep HBM
 //    traffic one-directional; at p = 1152 it beats column streaming up to
 //    the largest sizes;
-//  * otherwise column streaming once there are a quarter of the columns it
+//  * otherwise column streaming once there are a fifth of the columns it
 //    needs to fill the GPU (p = 36, 2x2 matrices, m = 2^16: 13 us against the
-//    tile's 15 us), and the shared-memory tile below that.
+//    tile's 15 us; 32768 int32 units: p = 64, 14.6 against 17.2 us, p = 127,
+//    28.4 against 32.5), and the shared-memory tile below that (8192 units:
+//    p = 64, 7.8 against 11.3 us; p = 127, 9.5 against 25.1).
 constexpr int64_t kTileMaxBytes = int64_t(40) << 20;
 constexpr int kSplitMinRanks = 128;
 constexpr int64_t kSplitWork = int64_t(1) << 17;
@@ -114,7 +116,7 @@ int fused_auto_mode(const Plan* P)
         return tile_beats_tree(P) ? 2 : 5;
     if (tile_preferred(P)) return 2;
     if (P->p >= kSplitMinRanks && units >= 4096 && P->split_ready) return 3;
-    if (units >= stream_target(P) / 4) return 1;
+    if (units >= stream_target(P) / 5) return 1;
     if (tile_lg_wu(P) >= 0) return 2;
     return P->split_ready ? 3 : 1;
 }
