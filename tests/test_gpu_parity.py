@@ -193,7 +193,10 @@ AUTO = [  # p, m, kind, layout the automatic choice takes on a 152-SM GPU
     # the shared-memory tile where it needs fewer waves of resident CTAs
     # than the hierarchical tile (p = 288: one against two)
     (288, 24576, "int32", 2), (288, 16384, "int32", 5), (576, 24576, "int32", 5),
-    (576, 32768, "int32", 5), (768, 24576, "int32", 5), (256, 28672, "int32", 2)]
+    (576, 32768, "int32", 5), (768, 24576, "int32", 5), (256, 28672, "int32", 2),
+    # below p = 128: column streaming from a fifth of the columns that fill
+    # the GPU (31129 units on 152 SMs), the shared-memory tile below
+    (64, 131072, "int32", 1), (64, 65536, "int32", 2)]
 
 
 @pytest.mark.parametrize("p,m,kind,mode", AUTO)
