@@ -313,6 +313,38 @@ def run_reference(args, w) -> dict:
                     "d2h_bytes_per_step": 0}}
 
 
+def run_oracle_sim(args) -> int:
+    """The oracle's event-level simulation of Algorithm 1 (every exchange of
+    every rank and round, with its unit-step clock) timed on one host core:
+    the two small workloads with their b, then the p = 1152 int32 sweep at
+    b = min(m, 16) while the next point would take under --cpu-seconds.  One JSON line
+    per point; CPU only, a reported baseline like cpu_baseline."""
+    import numpy as np
+    import torch
+    from oracle import oracle as O
+    from paper_2109_12626_gb300 import inputs as I
+    points = [("p7_m1000_int32", None), ("p36_m65536_mat2x2u32", None)]
+    points += [("p1152_int32_sweep", 1 << k) for k in range(0, 24, 2)]
+    for name, m in points:
+        w = workload(name, m)
+        p, kind, m = w["p"], w["kind"], w["m"]
+        kw = I.workload_kwargs(w)
+        x = torch.stack([I.rank_values(kind, w["seed"], i, m, **kw) for i in range(p)]).numpy()
+        dt = {"int32": O.I32, "float32": O.F32, "mat2x2u32": O.MAT, "mat2x2f32": O.MATF}[kind]
+        if kind == "mat2x2u32":
+            x = x.view(np.uint32).reshape(p, m, 4)
+        b = int(w.get("b") or min(m, 16))
+        t0 = time.perf_counter()
+        _, st, _ = O.simulate(x, dt, b)
+        el = time.perf_counter() - t0
+        print(json.dumps({"oracle_sim": name, "p": p, "m": m, "b": b, "seconds": round(el, 4),
+                          "ns_per_element": round(el * 1e9 / (p * m), 2), "cores": 1,
+                          "steps": st["steps"], "exchanges": st["exchanges"]}), flush=True)
+        if el * 4 > args.cpu_seconds:  # the next point is four times larger
+            break
+    return 0
+
+
 # -------------------------------------------------------------- sweeps
 def model_rounds(p: int, topology: str = "dual") -> int:
     """Unit steps before the first block reaches the last leaf in the
@@ -510,6 +542,8 @@ def main(argv=None) -> int:
                     help="e2e leg: 0 direct when possible, 1 copy pipeline, 2 direct")
     ap.add_argument("--transport", choices=tuple(TRANSPORTS), default="auto",
                     help="schedule kernel: how blocks pass between virtual ranks")
+    ap.add_argument("--oracle-sim", action="store_true",
+                    help="time the oracle's event-level simulation of Algorithm 1 (CPU)")
     args = ap.parse_args(argv)
     args.warmup = max(args.warmup, 3)
 
@@ -518,6 +552,8 @@ def main(argv=None) -> int:
     if args.p:
         w["p"] = int(args.p)
 
+    if args.oracle_sim:
+        return run_oracle_sim(args) if rank == 0 else 0
     if args.impl == "reference":
         if rank == 0:
             print(json.dumps(run_reference(args, w)), flush=True)

@@ -1,7 +1,7 @@
 """bench.py's host-side logic without a GPU: the max-over-ranks timing and
 barrier with two gloo ranks on the CPU (the N > 1 replica path), the clock
-sample parsing, the measured-traffic lookup, and the reference arm (the CPU
-oracle on a bounded sample)."""
+sample parsing, the measured-traffic lookup, the reference arm (the CPU
+oracle on a bounded sample) and the oracle-simulation timing leg."""
 import json
 import os
 import socket
@@ -92,6 +92,18 @@ def test_reference_arm_prints_one_json_line():
     assert d["impl"] == "reference" and d["unit"] == "GB/s" and d["value"] > 0
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] == 1
     assert d["e2e"]["h2d_bytes_per_step"] == 0
+
+
+def test_oracle_simulation_timing_leg():
+    """--oracle-sim times the oracle's event-level simulation of Algorithm 1
+    on the small workloads and stops the sweep at its time bound."""
+    out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--oracle-sim",
+                          "--cpu-seconds", "0.05"], capture_output=True, text=True, timeout=300)
+    assert out.returncode == 0, out.stderr
+    rows = [json.loads(l) for l in out.stdout.splitlines() if l.strip()]
+    assert [r["oracle_sim"] for r in rows[:2]] == ["p7_m1000_int32", "p36_m65536_mat2x2u32"]
+    assert rows[0]["b"] == 4 and rows[0]["steps"] > 0 and rows[0]["cores"] == 1
+    assert len(rows) < 14  # stopped before the largest sweep points
 
 
 def test_cost_model_fit_recovers_known_constants():
