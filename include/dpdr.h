@@ -152,8 +152,9 @@ int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
  *                             5 hierarchical tile (the five layouts of
  *                             dpdr_allreduce; 3 needs p >= 2 and keeps
  *                             m * esize bytes of scratch per subtree; 4 and
- *                             5 need 16-byte aligned buffers and otherwise
- *                             run as 1)
+ *                             5 need 16-byte aligned buffers: otherwise 4
+ *                             runs as 1, and 5 as 2, or as 3 (else 1) when
+ *                             a tile row of p elements does not fit)
  *   DPDR_OPT_WAIT_LIMIT_NS    bound of every wait of the schedule kernel,
  *                             nanoseconds (default 4e9)
  *   DPDR_OPT_SKIP_RANK        fault injection for tests: this rank of the
