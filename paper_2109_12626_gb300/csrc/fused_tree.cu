@@ -18,9 +18,10 @@
 // layout pays for a second kernel and a top fold per store group.  A CTA
 // reads all p rows of its columns before it writes any (barrier between
 // phases 1 and 3), and no other CTA touches those columns, so in-place use
-// is safe.  Buffers that are not all 16-byte aligned go to the streaming
-// layout; a ragged tail of single elements (fewer than 16 bytes per rank)
-// gets one extra CTA that runs the same three phases on them.
+// is safe.  Buffers that are not all 16-byte aligned go to the
+// shared-memory tile (fused.cu); a ragged tail of single elements (fewer
+// than 16 bytes per rank) gets one extra CTA that runs the same three
+// phases on them.
 #include <algorithm>
 #include <vector>
 
