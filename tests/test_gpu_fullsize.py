@@ -130,3 +130,34 @@ def test_p1152_int32_sweep(pkg, orc, m):
             _sampled_check(orc, w, m, xs, ys, _columns(m, b) if m > 4096 else np.arange(m))
     del xs, ys
     torch.cuda.empty_cache()
+
+
+def test_more_than_2_31_elements_per_rank(pkg, orc):
+    """m = 2^31 + 19 int32 per rank (8.6 GB each, p = 3): element and byte
+    offsets past 2^31 and 2^33, every fused layout that takes p = 3 and the
+    schedule kernel with both transports' block sizes, checked on sampled
+    columns around those boundaries and at random."""
+    w = dict(I.WORKLOADS["p7_m1000_int32"])
+    w["p"], m = 3, (1 << 31) + 19
+    dev = torch.device("cuda:0")
+    xs = _device_inputs(w, m, dev)
+    ys = [torch.empty_like(x) for x in xs]
+    with pkg.Plan(3, m, "int32", 0) as plan:
+        b = plan.query()["b"]
+        cols = _columns(m, b, k=4096)
+        edges = [c for e in ((1 << 31) - 1, 1 << 31, (1 << 31) + 16) for c in range(e - 3, e + 4)
+                 if c < m]
+        cols = np.unique(np.concatenate([cols, np.array(edges, np.int64)]))
+        for run, mode in (("fused", 0), ("fused", 2), ("fused", 4), ("fused", 5),
+                          ("schedule", 0)):
+            for y in ys:
+                y.fill_(-1)
+            if run == "fused":
+                plan.set(pkg.OPT_FUSED_MODE, mode)
+                plan.allreduce(xs, ys)
+            else:
+                plan.allreduce_schedule(xs, ys)
+            plan.sync()
+            _sampled_check(orc, w, m, xs, ys, cols)
+    del xs, ys
+    torch.cuda.empty_cache()
