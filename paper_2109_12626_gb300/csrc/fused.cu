@@ -109,11 +109,28 @@ static bool tile_preferred(const Plan* P)
            int64_t(P->p) * P->m * P->esize <= kTileMaxBytes;
 }
 
+// Beyond p = 2048 a wide hierarchical tile is long (walks of p / 32 ranks),
+// so a second wave of them that is less than 60 % full costs more than the
+// split layout's two kernels (p = 4094, m = 24576 int32: 166 against 181 us;
+// p = 8190, m = 20480: 282 against 322; p = 2304, m = 20480: 94 against
+// 110); with a fuller second wave the tile leads again (p = 4094, m = 2^15:
+// 186 against 194), and at p = 1152 it leads or ties throughout.
+static bool split_over_tree(const Plan* P)
+{
+    if (P->p < 2048 || fused_tree_index(P) != 1) return false;
+    const int64_t units = P->m * int64_t(P->esize) / 16;
+    const int64_t slots = int64_t(fused::kTreeCtasPerSm) * P->num_sms;
+    const int64_t ctas = (units + fused::kTreeUnitsWide - 1) / fused::kTreeUnitsWide;
+    return ctas > slots && (ctas - slots) * 10 < slots * 6;
+}
+
+static bool split_beats_tree(const Plan* P) { return P->split_ready && split_over_tree(P); }
+
 int fused_auto_mode(const Plan* P)
 {
     const int64_t units = P->m * int64_t(P->esize) / 16;
     if (P->tree[fused_tree_index(P)].ready && tree_preferred(P))
-        return tile_beats_tree(P) ? 2 : 5;
+        return tile_beats_tree(P) ? 2 : split_beats_tree(P) ? 3 : 5;
     if (tile_preferred(P)) return 2;
     if (P->p >= kSplitMinRanks && units >= 4096 && P->split_ready) return 3;
     if (units >= stream_target(P) / 5) return 1;
@@ -126,7 +143,8 @@ int fused_auto_mode(const Plan* P)
 static bool split_wanted(const Plan* P)
 {
     const int64_t units = P->m * int64_t(P->esize) / 16;
-    return P->p >= kSplitMinRanks && units >= 4096 && !tile_preferred(P) && !tree_preferred(P);
+    return P->p >= kSplitMinRanks && units >= 4096 && !tile_preferred(P) &&
+           (!tree_preferred(P) || split_over_tree(P));
 }
 
 // Split layout: cut depth s, subtree table, top-of-tree item list, rank

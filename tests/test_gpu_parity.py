@@ -196,7 +196,11 @@ AUTO = [  # p, m, kind, layout the automatic choice takes on a 152-SM GPU
     (576, 32768, "int32", 5), (768, 24576, "int32", 5), (256, 28672, "int32", 2),
     # below p = 128: column streaming from a fifth of the columns that fill
     # the GPU (31129 units on 152 SMs), the shared-memory tile below
-    (64, 131072, "int32", 1), (64, 65536, "int32", 2)]
+    (64, 131072, "int32", 1), (64, 65536, "int32", 2),
+    # from p = 2048 the split layout where the wide hierarchical tile's second
+    # wave would be less than 60 % full
+    (4094, 24576, "int32", 3), (4094, 32768, "int32", 5), (2304, 20480, "int32", 3),
+    (1152, 24576, "int32", 5)]
 
 
 @pytest.mark.parametrize("p,m,kind,mode", AUTO)
