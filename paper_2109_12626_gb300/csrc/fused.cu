@@ -1,6 +1,7 @@
 // fused.cu -- layout choice and launch of the fused bandwidth kernel
 // (dpdr_allreduce); the layouts themselves live in fused_stream.cu,
-// fused_tile.cu, fused_split.cu and fused_bulk.cu (see fused_common.cuh).
+// fused_tile.cu, fused_split.cu, fused_bulk.cu and fused_tree.cu (see
+// fused_common.cuh).
 #include <algorithm>
 #include <map>
 #include <mutex>
