@@ -437,7 +437,7 @@ def _stats(ts):
 
 def run_sweep(args, w) -> int:
     """--sweep m: every m = 2^0 .. 2^k of the workload, fused kernel (its
-    automatic layout) and schedule kernel (its automatic transport) at the
+    automatic layout, or --mode) and schedule kernel (its automatic transport) at the
     block-count rule, both timed as CUDA-graph replays of one call each (host
     launch overhead excluded): mean, min and median over the replays.  --sweep b: the schedule
     kernel's time against b at one m, with the Sec. 1.2 cost model fitted.
@@ -460,13 +460,15 @@ def run_sweep(args, w) -> int:
             b0 = -(-m // args.block_size) if args.block_size else 0
             with pkg.Plan(p, m, kind, b0, topology=args.topology) as plan:
                 plan.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[args.transport])
+                if args.mode:
+                    plan.set(pkg.OPT_FUSED_MODE, args.mode)
                 bd = plan.bind(xs, ys)
                 st = _stats(_timed_reps(lambda: bd.allreduce(), 20))
                 info = plan.info()
+                mode = args.mode or info["auto_mode"]
                 rec["fused"] = dict(st, gbs=round(2 * p * m * es / (st["us"] * 1e-6) / 1e9, 2),
-                                    layout=LAYOUTS[info["auto_mode"]],
-                                    split_depth=info["split_depth"] if info["auto_mode"] == 3
-                                    else None)
+                                    layout=LAYOUTS[mode],
+                                    split_depth=info["split_depth"] if mode == 3 else None)
                 st = _stats(_timed_reps(lambda: bd.allreduce_schedule(),
                                         5 if m >= (1 << 20) else 20))
                 plan.sync()

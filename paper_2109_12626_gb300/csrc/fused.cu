@@ -53,7 +53,10 @@ static int64_t stream_target(const Plan* P) { return int64_t(P->num_sms) * 1024;
 //    19.3 and 21.7; with as many waves the hierarchical tile is ahead or
 //    level: p = 256, m = 2^15, 17.5/20.8 against 19.8/26.3);
 //  * deep trees whose p input rows total at most kTileMaxBytes: the
-//    shared-memory tile, the layout with the lowest fixed cost (p = 192,
+//    shared-memory tile, the layout with the lowest fixed cost, in tiles
+//    narrowed until one wave of resident CTAs holds them when the columns
+//    are few (p = 288, m = 256 int32: 5.6/8.1 us warm/cold against 9.3/16.2
+//    at full width; p = 192,
 //    m = 2^15 int32: 11.4 us against the split layout's 19.9 us and the
 //    hierarchical tile's 17.7 us; at 75.5 MB the split layout wins at
 //    p = 288, 576 and 1152);
@@ -70,6 +73,13 @@ constexpr int64_t kTileMaxBytes = int64_t(40) << 20;
 constexpr int kSplitMinRanks = 128;
 constexpr int64_t kSplitWork = int64_t(1) << 17;
 constexpr int64_t kTreeMinBytesLargeP = int64_t(20) << 20;
+// Below p = 1024, up to this many column units the shared-memory tile, cut
+// into as many narrow tiles as one wave holds, beats the hierarchical tile
+// (p = 288, m = 1024 int32: 6.1/8.3 us warm/cold against 6.5/8.4; p = 576,
+// m = 4096: 8.5/12.0 against 11.0/12.3; p = 128, m = 2048: 5.0/6.3
+// against 6.2/8.2); above it the hierarchical tile leads cold (p = 576,
+// m = 8192: 14.5 against 17.0 us).
+constexpr int64_t kTileOverTreeUnits = 1024;
 
 // Resident CTAs of the shared-memory tile on the GPU: up to 4 per SM (256
 // threads of 64 registers), fewer when its rows do not fit the 228 KB of
@@ -86,7 +96,8 @@ static bool tree_preferred(const Plan* P)
     const int64_t units = P->m * int64_t(P->esize) / 16;
     const int64_t bytes = int64_t(P->p) * P->m * P->esize;
     if (units > (P->p >= 256 ? 8192 : 4096)) return false;
-    return P->p < 1024 || bytes > kTreeMinBytesLargeP;
+    if (P->p < 1024) return units > kTileOverTreeUnits;
+    return bytes > kTreeMinBytesLargeP;
 }
 
 // Whether the shared-memory tile needs fewer waves of resident CTAs than
@@ -239,6 +250,13 @@ int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t m
     const TreeTables& T = P->tree[tree_index < 0 ? fused_tree_index(P) : tree_index];
     if (mode == 5 && !T.ready) return fail(DPDR_ERR_INVALID, "tree mode not prepared");
     if (mode < 1 || mode > 5) return fail(DPDR_ERR_INVALID, "unknown fused mode");
+    // the bulk and hierarchical layouts need 16-byte rows: without them the
+    // bulk layout's work goes to column streaming, the hierarchical tile's to
+    // the shared-memory tile (or, when a tile row does not fit, the split
+    // layout), which keep its short walks (p = 288, m = 21250 int32 with
+    // rows 8 bytes apart from 16: 22.8 against 57 us streamed)
+    if (mode == 4 && !vec) mode = 1;
+    if (mode == 5 && !vec) mode = lg >= 0 ? 2 : P->split_ready ? 3 : 1;
 
     FusedArgs a;
     a.x = dx;
@@ -256,6 +274,17 @@ int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t m
     a.scalar_base = a.nvec * epv;
     a.nscalar = mc - a.scalar_base;
     a.lg_wu = lg < 0 ? 0 : lg;
+    if (mode == 2) {
+        // few columns: narrower tiles, as many as one wave of resident CTAs
+        // holds, so that each CTA copies fewer rank rows
+        const int sc = P->esize == 4 ? 2 : 0;  // single elements per 16 bytes, log2
+        auto tiles = [&](int l) {
+            return ((a.nvec + (int64_t(1) << l) - 1) >> l) +
+                   ((a.nscalar + (int64_t(1) << (l + sc)) - 1) >> (l + sc));
+        };
+        const int64_t slots = tile_slots(P);  // at the widest tile: a lower bound
+        while (a.lg_wu > 0 && tiles(a.lg_wu - 1) <= slots) a.lg_wu--;
+    }
     a.vec_tiles = (a.nvec + (int64_t(1) << a.lg_wu) - 1) >> a.lg_wu;
     a.seg = P->d_seg;
     a.items = P->d_items;
@@ -278,13 +307,6 @@ int fused_launch_cols(Plan* P, const char* const* dx, char* const* dy, int64_t m
     a.tree_slots = T.slots;
     a.tree_width = T.width;
     a.tree_tiles = T.width ? (a.nvec + T.width - 1) / T.width : 0;
-    // the bulk and hierarchical layouts need 16-byte rows: without them the
-    // bulk layout's work goes to column streaming, the hierarchical tile's to
-    // the shared-memory tile (or, when a tile row does not fit, the split
-    // layout), which keep its short walks (p = 288, m = 21250 int32 with
-    // rows 8 bytes apart from 16: 22.8 against 57 us streamed)
-    if (mode == 4 && !vec) mode = 1;
-    if (mode == 5 && !vec) mode = lg >= 0 ? 2 : P->split_ready ? 3 : 1;
 
     switch (mode) {
     case 1: return fused::launch_stream(P, a, s);

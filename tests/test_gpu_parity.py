@@ -187,6 +187,7 @@ AUTO = [  # p, m, kind, layout the automatic choice takes on a 152-SM GPU
           # (1 stream, 2 tile, 3 split, 5 hierarchical tile)
     (32, 1 << 27, "float32", 1), (36, 65536, "mat2x2u32", 1), (7, 1000, "int32", 2),
     (1152, 4096, "int32", 2), (1152, 8192, "int32", 5), (1152, 32768, "int32", 5),
+    (288, 4096, "int32", 2), (288, 4100, "int32", 5), (768, 4096, "int32", 2),
     (1152, 32772, "int32", 3), (128, 16384, "float32", 5), (192, 32768, "int32", 2),
     (288, 32768, "int32", 5), (288, 65536, "int32", 3), (4094, 2048, "int32", 5),
     (1152, 1 << 22, "float32", 3),
