@@ -138,6 +138,13 @@ DTYPES = {"int32": DPDR_INT32, "float32": DPDR_FLOAT32,
           "mat2x2u32": DPDR_MAT2X2_U32, "mat2x2f32": DPDR_MAT2X2_F32}
 
 
+# dpdr_plan_info's entries, in the header's order
+INFO_KEYS = ("p", "m", "b", "max_depth", "auto_mode", "sched_ctas",
+             "sched_ranks_per_cta", "scratch_bytes", "vector_path",
+             "split_depth", "split_subtrees", "split_group", "sched_slices",
+             "topology", "host_path", "sched_transport", "tree_width")
+
+
 class Plan:
     """A plan for p virtual ranks of m elements (``dpdr_plan``)."""
 
@@ -183,14 +190,10 @@ class Plan:
         return out
 
     def info(self) -> dict:
-        v = np.zeros(17, np.int64)
-        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), 17),
-               "dpdr_plan_info")
-        keys = ("p", "m", "b", "max_depth", "auto_mode", "sched_ctas",
-                "sched_ranks_per_cta", "scratch_bytes", "vector_path",
-                "split_depth", "split_subtrees", "split_group", "sched_slices",
-                "topology", "host_path", "sched_transport", "tree_width")
-        return {k: int(x) for k, x in zip(keys, v)}
+        n = len(INFO_KEYS)
+        v = np.zeros(n, np.int64)
+        _check(lib().dpdr_plan_info(self._h, v.ctypes.data_as(_I64P), n), "dpdr_plan_info")
+        return {k: int(x) for k, x in zip(INFO_KEYS, v)}
 
     def set(self, key: int, value: int) -> None:
         _check(lib().dpdr_plan_set(self._h, int(key), int(value)), "dpdr_plan_set")

@@ -123,3 +123,15 @@ def test_header_is_iso_c99_and_a_c_program_links(native, tmp_path):
     r, exe = c_build.build_program(str(tmp_path))
     assert r.returncode == 0, r.stderr
     assert os.path.exists(exe)
+
+
+def test_info_keys_follow_the_header():
+    """The binding names one key per entry dpdr.h documents for
+    dpdr_plan_info, no more and no fewer."""
+    import re
+    from paper_2109_12626_gb300 import _native as N
+    h = open(os.path.join(ROOT, "include", "dpdr.h")).read()
+    doc = h[h.index("Plan facts for tools and tests"):h.index("int dpdr_plan_info(")]
+    idx = sorted({int(k) for k in re.findall(r"\[(\d+)\]", doc)})
+    assert idx == list(range(len(N.INFO_KEYS)))
+
