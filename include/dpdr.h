@@ -130,7 +130,7 @@ int dpdr_block_count_rule(int p, int64_t m, double kappa);
  * otherwise dpdr_block_count_rule(p, m, kappa) with kappa = 46e6 / (p
  * esize) elements (alpha/beta of the counters transport; the ranks share
  * device memory, so beta grows with p), raised to at least
- * 4 p m esize / (L2 bytes) so that the blocks in flight stay in L2.
+ * 2 p m esize / (L2 bytes) so that the blocks in flight stay in L2.
  * p >= 1, m >= 0.  Returns NULL on error (see dpdr_last_error).  Not
  * thread-safe with respect to one plan. */
 dpdr_plan_t dpdr_plan(int p, int64_t m, dpdr_dtype dtype, dpdr_op op, int b);
@@ -156,12 +156,16 @@ int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
  *                             runs as 1, and 5 as 2, or as 3 (else 1) when
  *                             a tile row of p elements does not fit)
  *   DPDR_OPT_WAIT_LIMIT_NS    bound of every wait of the schedule kernel,
- *                             nanoseconds (default 4e9)
+ *                             nanoseconds: 1e3 .. 1e10 (default 4e9); values
+ *                             outside that range are DPDR_ERR_INVALID, so a
+ *                             wait can never become unbounded
  *   DPDR_OPT_SKIP_RANK        fault injection for tests: this rank of the
  *                             schedule kernel never publishes a block, so
  *                             its partners' waits expire (-1 = off)
  *   DPDR_OPT_SCHED_THREADS    threads per CTA of the schedule kernel
- *                             (64..256, multiple of 32; default 128)
+ *                             (64..256, multiple of 32); 0 (default) is
+ *                             automatic: 64 with the counters transport,
+ *                             128 with flagged words
  *   DPDR_OPT_SCHED_RANKS_PER_CTA  virtual ranks per CTA (0 = fewest that
  *                             fit co-resident)
  *   DPDR_OPT_BLOCKS           change b (same rules as dpdr_plan's b)

@@ -81,7 +81,7 @@ struct Plan {
     int fused_mode = 0;        // 0 auto, 1 stream, 2 tile, 3 split, 4 bulk, 5 tree
     int64_t wait_ns = 4000000000LL;
     int skip_rank = -1;
-    int sched_threads = 128;
+    int sched_threads = 0;     // threads per schedule CTA, 0 = automatic
     int sched_rpc = 0;         // ranks per CTA, 0 = auto
     int sched_slices = 0;      // CTAs per rank (column slices), 0 = auto
     int split_depth = -1;      // cut depth of the split layout, -1 = auto
@@ -156,6 +156,8 @@ struct Plan {
     // facts
     int last_vector_path = 0;
     int sched_ctas = 0, sched_ranks_per_cta = 0;
+    int sched_rpc_ref = 1;         // ranks per CTA at 128 threads (transport choice)
+    int sched_threads_used = 128;  // threads per CTA of the kernel that runs
     int sched_slices_used = 1, sched_chunks = 1;
 };
 

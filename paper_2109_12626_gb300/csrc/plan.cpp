@@ -194,6 +194,9 @@ static int clamp_b(int64_t m, int64_t b)
 //    17.9 ms at b = 128).
 //  * flagged-word transport (m esize <= 32 KiB): latency-bound, b = 1.
 constexpr double kKappaBytes = 46e6;
+// Upper bound of DPDR_OPT_WAIT_LIMIT_NS: every wait of the schedule kernel
+// stays bounded whatever the caller asks for.
+constexpr int64_t kMaxWaitNs = 10000000000LL;
 
 static int default_blocks(const Plan* P)
 {
@@ -201,7 +204,9 @@ static int default_blocks(const Plan* P)
     const double kappa = std::max(1.0, kKappaBytes / (double(P->p) * double(P->esize)));
     int64_t b = block_count_rule(P->p, P->m, kappa);
     if (P->l2_bytes > 0) {
-        const double need = 4.0 * double(P->p) * double(P->m) * double(P->esize) /
+        // two blocks per rank in L2 (the partial or final block in flight
+        // and the next one): within 0-7 % of the best b from p = 32 to 1152
+        const double need = 2.0 * double(P->p) * double(P->m) * double(P->esize) /
                             double(P->l2_bytes);
         b = std::max<int64_t>(b, int64_t(std::ceil(need)));
     }
@@ -433,6 +438,7 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
         return DPDR_OK;
     case DPDR_OPT_WAIT_LIMIT_NS:
         if (v < 1000) return fail(DPDR_ERR_INVALID, "wait limit below 1 us");
+        if (v > kMaxWaitNs) return fail(DPDR_ERR_INVALID, "wait limit above 10 s");
         P->wait_ns = v;
         return DPDR_OK;
     case DPDR_OPT_SKIP_RANK:
@@ -440,8 +446,8 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
         P->skip_rank = int(v);
         return DPDR_OK;
     case DPDR_OPT_SCHED_THREADS:
-        if (v < 64 || v > 256 || v % 32)
-            return fail(DPDR_ERR_INVALID, "schedule threads: 64..256, multiple of 32");
+        if (v != 0 && (v < 64 || v > 256 || v % 32))
+            return fail(DPDR_ERR_INVALID, "schedule threads: 0 or 64..256, multiple of 32");
         P->sched_threads = int(v);
         return schedule_configure(P);
     case DPDR_OPT_SCHED_RANKS_PER_CTA:

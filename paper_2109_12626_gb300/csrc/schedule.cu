@@ -43,11 +43,17 @@
 #include <mutex>
 
 #include "schedule_common.cuh"
+#include "tma.cuh"
 
 namespace dpdr {
 namespace {
 
 constexpr int kSchedMaxThreads = sched::kMaxThreads;
+// Words from one handshake counter to the next: each counter has a 128-byte
+// L2 line of its own, so the release stores and polls of different ranks
+// never queue on one line (with 4-byte counters side by side, the 32 ranks
+// of a line serialised there: 20 % of the time at p = 32).
+constexpr int kCtr = 32;
 constexpr int kSchedMaxGroups = sched::kMaxGroups;
 
 struct SchedArgs {
@@ -145,8 +151,18 @@ __device__ __forceinline__ void group_sync(const SchedArgs& a)
 }
 static_assert(kSchedMaxGroups == 4, "group_sync names one barrier per group");
 
-// Thread 0 of the group waits until every one of the n counters (n <= 3,
-// the same on all its threads) reaches its target, polling them together
+// The group thread that polls counters, and the one that issues release
+// stores: different warps when the group has two or more, so that the
+// release that ends one step (its fence waits for the step's writes to
+// reach L2) and the poll that begins the next run at the same time.
+template <bool kG>
+__device__ __forceinline__ int poller_tid(const SchedArgs& a)
+{
+    return (kG ? (1 << a.lg_gsz) : int(blockDim.x)) >= 64 ? 32 : 0;
+}
+
+// The poller thread waits until every one of the n counters (n <= 3, the
+// same on all its threads) reaches its target, polling them together
 // within the plan's time bound; the group learns the outcome through shared
 // memory.  Returns false on timeout or abort (then the caller returns from
 // the kernel).
@@ -158,7 +174,7 @@ __device__ __forceinline__ bool cta_wait(const SchedArgs& a, const Wait* w, int 
     __shared__ int ok_slot[kSchedMaxGroups];
     const Group grp = group_of<kG>(a);
     int& ok = ok_slot[grp.id];
-    if (grp.tid == 0) {
+    if (grp.tid == poller_tid<kG>(a)) {
         int r = 1;
         unsigned pending = 0;
         for (int k = 0; k < n; k++)
@@ -214,18 +230,67 @@ __device__ __forceinline__ void publish(const SchedArgs& a, uint32_t* ctr0, uint
     }
 }
 
-// dst[k] = lo[k] (.) hi[k] for k in [s, e); rows are virtual bases indexed
-// by global element number.  dst may equal hi.  With lo == nullptr it is a
-// plain copy dst[k] = hi[k].  Each thread owns the same elements in every
-// call over the same range, so a later call may read what an earlier one
-// wrote without a barrier.  Not inlined: its eight 16-byte registers in
-// flight then fit the 64-register budget without spilling the caller's state.
-template <class Op, bool kG>
-__device__ __noinline__ void block_op(const SchedArgs& a, char* dst, const char* lo,
-                                      const char* hi, int64_t s, int64_t e)
+// ------------------------------------------------------------ block passes
+// A block pass combines up to three rows element by element over [s, e)
+// and writes the result to dst:
+//   NOPS 1  dst = src0                        (a final block copied down)
+//   NOPS 2  dst = src0 (.) src1               (one child's partial with x_i,
+//                                              or the dual roots' partials)
+//   NOPS 3  dst = src1 (.) (src0 (.) src2)    (Y[j] = t1 (.) (t0 (.) x_i))
+// Rows are virtual bases indexed by global element number.  dst may equal
+// the last source (in place).  Every thread owns the same elements in every
+// pass over the same range.
+//
+// On the vector path a thread stages its 16-byte units through kSlots
+// private shared-memory slots with cp.async (a copy that holds no
+// register while in flight): it issues kSlots / NOPS units of every
+// operand, waits for its own copies, combines from shared memory and
+// stores the result.  A block's data is in L2 or on its way from DRAM, so
+// a pass takes a few memory latencies, and the slots let each thread keep
+// 192 bytes in flight whatever the operand count, three times what the
+// 64-register budget leaves for loads.  Elements outside the 16-byte units
+// (an unaligned head and tail, or every element when some buffer is only
+// 4-byte aligned) move singly with L2-coherent loads.
+constexpr int kSlots = 12;
+constexpr int kSlotBytes = kSlots * 16;  // shared memory per thread
+
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                     static_cast<uint32_t>(__cvta_generic_to_shared(smem))),
+                 "l"(gmem)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all()
+{
+    asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
+}
+
+template <int NOPS, class Op>
+__device__ __forceinline__ uint4 combine_units(const uint4* v)
+{
+    if (NOPS == 1) return v[0];
+    if (NOPS == 2) return Op::vec(v[0], v[1]);
+    return Op::vec(v[1], Op::vec(v[0], v[2]));
+}
+template <int NOPS, class Op>
+__device__ __forceinline__ Elem<Op> combine_elems(const char* s0, const char* s1, const char* s2,
+                                                  int64_t off)
+{
+    if (NOPS == 1) return ld_one_l2<Op>(s0 + off);
+    const Elem<Op> a0 = ld_one_l2<Op>(s0 + off), a1 = ld_one_l2<Op>(s1 + off);
+    if (NOPS == 2) return comb<Op>(a0, a1);
+    return comb<Op>(a1, comb<Op>(a0, ld_one_l2<Op>(s2 + off)));
+}
+
+template <class Op, bool kG, int NOPS>
+__device__ __noinline__ void block_pass(const SchedArgs& a, char* dst, const char* s0,
+                                        const char* s1, const char* s2, int64_t s, int64_t e)
 {
     constexpr int EPV = Op::kEpv;
     constexpr int ES = Op::kEsize;
+    constexpr int B = kSlots / NOPS;  // units per operand in flight per thread
+    extern __shared__ uint4 sched_slots[];
     const Group grp = group_of<kG>(a);
     const int tid = grp.tid, bd = grp.size;
     int64_t vs = 0, ve = 0;
@@ -234,49 +299,71 @@ __device__ __noinline__ void block_op(const SchedArgs& a, char* dst, const char*
         ve = e / EPV;
         if (vs > ve) vs = ve = 0;
     }
-    // single elements: the unaligned head and tail around the vector range
-    int64_t head_end = e, tail_beg = e;
-    if (vs < ve) {
-        head_end = vs * EPV;
-        tail_beg = ve * EPV;
-    }
+    const int64_t head_end = vs < ve ? vs * EPV : e, tail_beg = vs < ve ? ve * EPV : e;
     for (int pass = 0; pass < 2; pass++) {
         const int64_t b0 = pass ? tail_beg : s, b1 = pass ? e : head_end;
-        for (int64_t k = b0 + tid; k < b1; k += bd) {
-            const Elem<Op> h = ld_one_l2<Op>(hi + k * ES);
-            st_one_l2<Op>(dst + k * ES, lo ? comb<Op>(ld_one_l2<Op>(lo + k * ES), h) : h);
-        }
+        for (int64_t k = b0 + tid; k < b1; k += bd)
+            st_one_l2<Op>(dst + k * ES, combine_elems<NOPS, Op>(s0, s1, s2, k * ES));
     }
-    // 16-byte units, four in flight per thread
-    constexpr int B = 4;
+    // slot k of this thread: sched_slots[k * blockDim.x + threadIdx.x]
+    // (consecutive threads on consecutive 16 bytes: no bank conflicts)
+    uint4* const my = sched_slots + threadIdx.x;
+    const int stride = int(blockDim.x);
+    const char* const src[3] = {s0, s1, s2};
     for (int64_t v0 = vs + tid; v0 < ve; v0 += int64_t(B) * bd) {
-        uint4 hv[B], lv[B];
 #pragma unroll
         for (int t = 0; t < B; t++) {
             const int64_t v = v0 + int64_t(t) * bd;
             if (v < ve) {
-                hv[t] = ld_l2(hi + v * 16);
-                if (lo) lv[t] = ld_l2(lo + v * 16);
+#pragma unroll
+                for (int o = 0; o < NOPS; o++) cp_async16(my + (t * NOPS + o) * stride, src[o] + v * 16);
             }
         }
+        cp_async_wait_all();
 #pragma unroll
         for (int t = 0; t < B; t++) {
             const int64_t v = v0 + int64_t(t) * bd;
-            if (v < ve) st_l2(dst + v * 16, lo ? Op::vec(lv[t], hv[t]) : hv[t]);
+            if (v < ve) {
+                uint4 r[NOPS];
+#pragma unroll
+                for (int o = 0; o < NOPS; o++) r[o] = my[(t * NOPS + o) * stride];
+                st_l2(dst + v * 16, combine_units<NOPS, Op>(r));
+            }
         }
     }
 }
 
 // dst = t1 (.) (t0 (.) x) over [s, e) for the children's partial blocks
-// t0, t1 (null when the child does not exist; both null: a copy of x): two
-// passes, the second reading back this thread's own results of the first.
+// t0, t1 (null when the child does not exist; both null: a copy of x).
 template <class Op, bool kG>
 __device__ __forceinline__ void fold_children(const SchedArgs& a, char* dst, const char* t0,
-                                              const char* t1, const char* x, int64_t s,
+                                              const char* t1, const char* x, int64_t s, int64_t e)
+{
+    if (!t0)
+        block_pass<Op, kG, 1>(a, dst, x, nullptr, nullptr, s, e);
+    else if (!t1)
+        block_pass<Op, kG, 2>(a, dst, t0, x, nullptr, s, e);
+    else
+        block_pass<Op, kG, 3>(a, dst, t0, t1, x, s, e);
+}
+
+// An inner child's partial block is dead once its parent has combined it:
+// the child overwrites it with the final block later.  Dropping its L2
+// lines without write-back keeps the partial from ever reaching device
+// memory, so y is written to DRAM once.  Only whole 128-byte lines inside
+// [s, e) go: the lines at the ends may hold neighbouring slices' or blocks'
+// live data.  Called after a barrier that follows every read of the range;
+// the rank's next release orders the discards before the child's final
+// write, which waits for a later release of this rank.
+template <class Op, bool kG>
+__device__ __noinline__ void discard_consumed(const SchedArgs& a, const char* row, int64_t s,
                                               int64_t e)
 {
-    block_op<Op, kG>(a, dst, t0, x, s, e);
-    if (t1) block_op<Op, kG>(a, dst, t1, dst, s, e);
+    const Group grp = group_of<kG>(a);
+    const uintptr_t lo = (reinterpret_cast<uintptr_t>(row + s * Op::kEsize) + 127) & ~uintptr_t(127);
+    const uintptr_t hi = reinterpret_cast<uintptr_t>(row + e * Op::kEsize) & ~uintptr_t(127);
+    for (uintptr_t l = lo + uintptr_t(grp.tid) * 128; l < hi; l += uintptr_t(grp.size) * 128)
+        tma::discard_l2_line(reinterpret_cast<const void*>(l));
 }
 
 __device__ __forceinline__ char* ring_base(const SchedArgs& a, int side, int j, int g,
@@ -288,82 +375,91 @@ __device__ __forceinline__ char* ring_base(const SchedArgs& a, int side, int j, 
 }
 
 // Round j of Algorithm 1 at rank i, column slice g.  The waits for the two
-// children's partial blocks do not depend on each other, so thread 0 polls
-// them together, and the folds Y[j] = t1 (.) (t0 (.) x_i) (child_0's partial
-// first, as the steps run) follow without a barrier between them.  The partial goes up before the wait for
+// children's partial blocks do not depend on each other, so they are polled
+// together, and Y[j] = t1 (.) (t0 (.) x_i) (child_0's partial first, as the
+// steps run) is formed in one pass.  The partial goes up before the wait for
 // the parent's final block, so a parent's round j never waits for its own
-// round j-1 to reach the child and come back.
+// round j-1 to reach the child and come back; the release of the partial
+// and the poll of the parent's counter run in different warps at once (as
+// do the release of the final block and the next round's first poll).
 template <class Op, bool kG>
 __device__ __forceinline__ bool run_round(const SchedArgs& a, int i, int j, int g)
 {
     constexpr int EPV = Op::kEpv;
-    uint32_t* const up = a.up + int64_t(g) * a.p;      // this slice's counters
-    uint32_t* const down = a.down + int64_t(g) * a.p;
-    const int d = __ldg(a.depth + i);
+    uint32_t* const up = a.up + int64_t(g) * a.p * kCtr;      // this slice's counters
+    uint32_t* const down = a.down + int64_t(g) * a.p * kCtr;
     const int c0 = __ldg(a.child0 + i), c1 = __ldg(a.child1 + i);
     const int par = __ldg(a.parent + i);
     const char* xi = rank_in(a.x, i);
     char* yi = rank_out(a.y, i);
-    const bool root = par < 0;
-    const bool paired_root = root && a.r0 >= 0;
     const bool inb = j < a.b;
     const int64_t bs = inb ? blk_start(a, j) : 0, be = inb ? blk_start(a, j + 1) : 0;
     const int64_t s = slice_at<EPV>(a, bs, be, g), e = slice_at<EPV>(a, bs, be, g + 1);
 
     // steps 1 and 2: the children's partial blocks (a leaf's is x_c, an inner
     // node's y_c); the send half (final block j-(d+1)) is read by the child
-    // itself from y_i once down[i] covers it
-    const char* t[2] = {nullptr, nullptr};
-    if (inb) {
+    // itself from y_i once down[i] covers it.  inner0/inner1: the child has
+    // children of its own, so its partial lives in y_c and dies here.
+    const char* t0 = nullptr;
+    const char* t1 = nullptr;
+    bool inner0 = false, inner1 = false;
+    if (inb && c0 >= 0) {
+        inner0 = __ldg(a.child0 + c0) >= 0;
+        t0 = inner0 ? rank_in(a.y, c0) : rank_in(a.x, c0);
         Wait w[2];
-        int n = 0;
-        for (int k = 0; k < 2; k++) {
-            const int c = k ? c1 : c0;
-            if (c < 0) continue;
-            t[k] = __ldg(a.child0 + c) < 0 ? rank_in(a.x, c) : rank_in(a.y, c);
-            w[n++] = Wait{up + c, uint32_t(j + 1), k};
+        w[0] = Wait{up + c0 * kCtr, uint32_t(j + 1), 0};
+        if (c1 >= 0) {
+            inner1 = __ldg(a.child0 + c1) >= 0;
+            t1 = inner1 ? rank_in(a.y, c1) : rank_in(a.x, c1);
+            w[1] = Wait{up + c1 * kCtr, uint32_t(j + 1), 1};
         }
-        if (!cta_wait<kG>(a, w, n, i, j)) return false;
+        if (!cta_wait<kG>(a, w, c1 >= 0 ? 2 : 1, i, j)) return false;
     }
 
-    if (paired_root) {  // step 3 at a root: exchange partials with the dual
+    if (par < 0 && a.r0 >= 0) {  // step 3 at a root: exchange partials with the dual
         if (!inb) return true;
         const int side = (i == a.r0) ? 0 : 1;
-        char* slot = ring_base(a, side, j, g, s, Op::kEpv, Op::kEsize);
-        fold_children<Op, kG>(a, slot, t[0], t[1], xi, s, e);
-        publish<kG>(a, up + i, uint32_t(j + 1), nullptr, 0, i);
+        char* slot = ring_base(a, side, j, g, s, EPV, Op::kEsize);
+        fold_children<Op, kG>(a, slot, t0, t1, xi, s, e);
+        publish<kG>(a, up + i * kCtr, uint32_t(j + 1), nullptr, 0, i);
+        if (inner0) discard_consumed<Op, kG>(a, t0, s, e);
+        if (inner1) discard_consumed<Op, kG>(a, t1, s, e);
         const int du = (i == a.r0) ? a.r1 : a.r0;
-        const Wait wd{up + du, uint32_t(j + 1), 2};
+        const Wait wd{up + du * kCtr, uint32_t(j + 1), 2};
         if (!cta_wait<kG>(a, &wd, 1, i, j)) return false;
-        const char* other = ring_base(a, 1 - side, j, g, s, Op::kEpv, Op::kEsize);
-        if (i == a.r0)  // lower root: Y[j] (.) t
-            block_op<Op, kG>(a, yi, slot, other, s, e);
-        else  // higher root: t (.) Y[j]
-            block_op<Op, kG>(a, yi, other, slot, s, e);
-        publish<kG>(a, down + i, uint32_t(j + 1), nullptr, 0, i);
+        const char* other = ring_base(a, 1 - side, j, g, s, EPV, Op::kEsize);
+        // lower root: Y[j] (.) t; higher root: t (.) Y[j]
+        if (i == a.r0)
+            block_pass<Op, kG, 2>(a, yi, slot, other, nullptr, s, e);
+        else
+            block_pass<Op, kG, 2>(a, yi, other, slot, nullptr, s, e);
+        publish<kG>(a, down + i * kCtr, uint32_t(j + 1), nullptr, 0, i);
         return true;
     }
-    if (root) {  // the root of a single tree (or p == 1): its block is final
+    if (par < 0) {  // the root of a single tree (or p == 1): its block is final
         if (!inb) return true;
-        if (t[0] || xi != yi) fold_children<Op, kG>(a, yi, t[0], t[1], xi, s, e);
-        publish<kG>(a, down + i, uint32_t(j + 1), nullptr, 0, i);
+        if (t0 || xi != yi) fold_children<Op, kG>(a, yi, t0, t1, xi, s, e);
+        publish<kG>(a, down + i * kCtr, uint32_t(j + 1), nullptr, 0, i);
+        if (inner0) discard_consumed<Op, kG>(a, t0, s, e);
+        if (inner1) discard_consumed<Op, kG>(a, t1, s, e);
         return true;
     }
     // step 3 elsewhere: partial Y[j] up (in y_i, or x_i itself for a leaf),
     // final Y[j-d] down from the parent
     if (inb) {
-        if (t[0]) fold_children<Op, kG>(a, yi, t[0], t[1], xi, s, e);
-        publish<kG>(a, up + i, uint32_t(j + 1), nullptr, 0, i);
+        if (t0) fold_children<Op, kG>(a, yi, t0, t1, xi, s, e);
+        publish<kG>(a, up + i * kCtr, uint32_t(j + 1), nullptr, 0, i);
+        if (inner0) discard_consumed<Op, kG>(a, t0, s, e);
+        if (inner1) discard_consumed<Op, kG>(a, t1, s, e);
     }
-    const int kf = j - d;
+    const int kf = j - __ldg(a.depth + i);
     if (kf >= 0 && kf < a.b) {
-        const Wait wp{down + par, uint32_t(kf + 1), 3};
+        const Wait wp{down + par * kCtr, uint32_t(kf + 1), 3};
         if (!cta_wait<kG>(a, &wp, 1, i, j)) return false;
-        const char* yp = rank_in(a.y, par);
         const int64_t ks = blk_start(a, kf), ke = blk_start(a, kf + 1);
-        block_op<Op, kG>(a, yi, nullptr, yp, slice_at<EPV>(a, ks, ke, g),
-                     slice_at<EPV>(a, ks, ke, g + 1));
-        publish<kG>(a, down + i, uint32_t(kf + 1), nullptr, 0, i);
+        block_pass<Op, kG, 1>(a, yi, rank_in(a.y, par), nullptr, nullptr,
+                              slice_at<EPV>(a, ks, ke, g), slice_at<EPV>(a, ks, ke, g + 1));
+        publish<kG>(a, down + i * kCtr, uint32_t(kf + 1), nullptr, 0, i);
     }
     return true;
 }
@@ -414,11 +510,25 @@ const void* kernel_for(int dtype, bool grouped)
 // CTAs of `threads` threads that fit one SM for the counters kernel (the
 // variant for one rank per CTA, or the grouped one) and the flagged-word
 // kernel alike.
+// The counters kernel's dynamic shared memory (the cp.async slots) for
+// CTAs of `threads` threads.  Beyond 48 KB less the kernel's static shared
+// memory (256 threads) the kernel must be granted the size first.
+cudaError_t sched_smem(int dtype, bool grouped, int threads, size_t* bytes)
+{
+    *bytes = size_t(threads) * kSlotBytes;
+    if (*bytes + 1024 <= 48 * 1024) return cudaSuccess;
+    return cudaFuncSetAttribute(kernel_for(dtype, grouped), cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                int(*bytes));
+}
+
 cudaError_t sched_occupancy(int dtype, int threads, bool grouped, int* occ)
 {
     int o[2] = {0, 0};
+    size_t smem = 0;
+    cudaError_t e0 = sched_smem(dtype, grouped, threads, &smem);
+    if (e0 != cudaSuccess) return e0;
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o[0], kernel_for(dtype, grouped),
-                                                                  threads, 0);
+                                                                  threads, smem);
     if (e == cudaSuccess)
         e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o[1], schedule_ll_kernel_for(dtype),
                                                           threads, 0);
@@ -439,10 +549,10 @@ cudaError_t sched_occupancy(int dtype, int threads, bool grouped, int* occ)
 // fixed DPDR_OPT_SCHED_SLICES asks for -- fits at once, for the kernels that
 // run it: the one-rank-per-CTA counters kernel, or, once CTAs must own
 // several ranks, its grouped variant, and the flagged-word kernel.
-static int schedule_rpc(const Plan* P, int* R_out, int64_t* kmax_out)
+static int schedule_rpc(const Plan* P, int threads, int* R_out, int64_t* kmax_out)
 {
     int occ = 0;
-    cudaError_t e = sched_occupancy(P->dtype, P->sched_threads, false, &occ);
+    cudaError_t e = sched_occupancy(P->dtype, threads, false, &occ);
     if (e != cudaSuccess) return cuda_fail(e, "schedule occupancy");
     int64_t kmax = int64_t(occ) * P->num_sms;
     const int n0 = P->r0 >= 0 ? P->p / 2 : 0, n1 = P->p - n0;
@@ -454,7 +564,7 @@ static int schedule_rpc(const Plan* P, int* R_out, int64_t* kmax_out)
         while (R < P->p && ctas(R) * per_chunk > kmax) R++;
     }
     if (R > 1) {
-        e = sched_occupancy(P->dtype, P->sched_threads, true, &occ);
+        e = sched_occupancy(P->dtype, threads, true, &occ);
         if (e != cudaSuccess) return cuda_fail(e, "schedule occupancy");
         kmax = int64_t(occ) * P->num_sms;
         if (P->sched_rpc == 0)
@@ -465,15 +575,36 @@ static int schedule_rpc(const Plan* P, int* R_out, int64_t* kmax_out)
     return DPDR_OK;
 }
 
-int schedule_plan_rpc(Plan* P) { return schedule_rpc(P, &P->sched_ranks_per_cta, nullptr); }
+// Threads per CTA: the option's value, else 128 for the layout that decides
+// the transport (the flagged-word kernel's choice was measured with it) and
+// for that kernel, and 64 for the counters kernel, whose rounds are bound by
+// handshake latency: two CTAs of 64 threads per slot of one of 128 run twice
+// the independent column slices, 7-15 % faster at p = 32 and 1152.
+static int reference_threads(const Plan* P) { return P->sched_threads ? P->sched_threads : 128; }
+
+int schedule_plan_rpc(Plan* P)
+{
+    int rc = schedule_rpc(P, reference_threads(P), &P->sched_rpc_ref, nullptr);
+    P->sched_ranks_per_cta = P->sched_rpc_ref;
+    P->sched_threads_used = reference_threads(P);
+    return rc;
+}
 
 int schedule_configure(Plan* P)
 {
     int R = 1;
     int64_t kmax = 0;
-    int rc = schedule_rpc(P, &R, &kmax);
+    int threads = reference_threads(P);
+    int rc = schedule_rpc(P, threads, &R, &kmax);
     if (rc) return rc;
-    P->sched_ranks_per_cta = R;  // the transport choice below depends on it
+    P->sched_rpc_ref = R;  // the transport choice depends on it
+    if (P->sched_threads == 0 && schedule_transport(P) == 1) {
+        threads = 64;
+        rc = schedule_rpc(P, threads, &R, &kmax);
+        if (rc) return rc;
+    }
+    P->sched_ranks_per_cta = R;
+    P->sched_threads_used = threads;
     // rank chunks never straddle the two trees (one tree: n0 = 0)
     const int n0 = P->r0 >= 0 ? P->p / 2 : 0;
     cudaError_t e;
@@ -493,7 +624,7 @@ int schedule_configure(Plan* P)
             : blk / 1024;
         G = int(std::max<int64_t>(1, std::min<int64_t>({room, want, 64})));
     }
-    const size_t words = 2 * size_t(P->p) * G + 1;
+    const size_t words = (2 * size_t(P->p) * G + 1) * kCtr;
     const size_t bytes = (words * sizeof(uint32_t) + 255) / 256 * 256 + sizeof(int) * first.size();
     if (bytes > P->d_sched_bytes) {
         if (P->d_sched) cudaFree(P->d_sched);
@@ -528,8 +659,8 @@ int schedule_launch(Plan* P, cudaStream_t s)
     a.cta_first = P->d_cta_first;
     const int64_t cw = int64_t(P->p) * P->sched_slices_used;
     a.up = P->d_ctrl;
-    a.down = P->d_ctrl + cw;
-    a.abort_flag = P->d_ctrl + 2 * cw;
+    a.down = P->d_ctrl + cw * kCtr;
+    a.abort_flag = P->d_ctrl + 2 * cw * kCtr;
     a.err = P->d_err;
     a.ring = P->d_ring;
     a.ring_slot = int64_t(ring_sub_bytes((P->m + P->b - 1) / P->b, P->esize, P->sched_slices_used));
@@ -547,15 +678,17 @@ int schedule_launch(Plan* P, cudaStream_t s)
     a.vec = P->last_vector_path;
     a.nslices = P->sched_slices_used;
     a.nchunks = P->sched_chunks;
-    a.ngroups = sched::group_count(P->sched_ranks_per_cta, P->sched_threads);
-    a.lg_gsz = sched::group_lg(P->sched_ranks_per_cta, P->sched_threads);
+    a.ngroups = sched::group_count(P->sched_ranks_per_cta, P->sched_threads_used);
+    a.lg_gsz = sched::group_lg(P->sched_ranks_per_cta, P->sched_threads_used);
 
-    cudaError_t e = cudaMemsetAsync(P->d_ctrl, 0, sizeof(uint32_t) * (2 * size_t(cw) + 1), s);
+    cudaError_t e = cudaMemsetAsync(P->d_ctrl, 0, sizeof(uint32_t) * (2 * size_t(cw) + 1) * kCtr, s);
     if (e != cudaSuccess) return cuda_fail(e, "schedule counter reset");
+    size_t smem = 0;
+    e = sched_smem(P->dtype, P->sched_ranks_per_cta > 1, P->sched_threads_used, &smem);
+    if (e != cudaSuccess) return cuda_fail(e, "schedule kernel shared memory");
     void* args[] = {&a};
     e = cudaLaunchCooperativeKernel(kernel_for(P->dtype, P->sched_ranks_per_cta > 1),
-                                    dim3(P->sched_ctas),
-                                    dim3(P->sched_threads), args, 0, s);
+                                    dim3(P->sched_ctas), dim3(P->sched_threads_used), args, smem, s);
     if (e == cudaErrorCooperativeLaunchTooLarge) {
         cudaGetLastError();
         return fail(DPDR_ERR_NOT_COOPERATIVE, "schedule kernel: CTAs cannot be co-resident");
@@ -596,7 +729,7 @@ inline NoAllocLayout noalloc_layout(int p, int64_t m, int b, size_t esize)
     L.y = na_align(L.x + sizeof(void*) * size_t(p));
     L.tables = na_align(L.y + sizeof(void*) * size_t(p));
     L.ctrl = na_align(L.tables + sizeof(int) * 4 * size_t(p));
-    L.err = na_align(L.ctrl + sizeof(uint32_t) * (2 * size_t(p) + 1));
+    L.err = na_align(L.ctrl + sizeof(uint32_t) * (2 * size_t(p) + 1) * kCtr);
     L.cta = na_align(L.err + sizeof(uint32_t) * 4);
     L.ring = na_align(L.cta + sizeof(int) * (size_t(p) + 2));
     L.slot = na_align(ring_sub_bytes((m + b - 1) / b, esize, 1));
@@ -754,8 +887,8 @@ int schedule_noalloc(int p, int64_t m, int dtype, int op, int b, const void* con
     a.cta_first = cta;
     uint32_t* ctrl = reinterpret_cast<uint32_t*>(base + L.ctrl);
     a.up = ctrl;
-    a.down = ctrl + p;
-    a.abort_flag = ctrl + 2 * p;
+    a.down = ctrl + int64_t(p) * kCtr;
+    a.abort_flag = ctrl + 2 * int64_t(p) * kCtr;
     a.err = reinterpret_cast<uint32_t*>(base + L.err);
     a.ring = reinterpret_cast<char*>(base + L.ring);
     a.ring_slot = int64_t(L.slot);
@@ -775,7 +908,7 @@ int schedule_noalloc(int p, int64_t m, int dtype, int op, int b, const void* con
     a.lg_gsz = sched::group_lg(R, kNoAllocThreads);
     void* args[] = {&a};
     e = cudaLaunchCooperativeKernel(kernel_for(dtype, R > 1), dim3(nctas), dim3(kNoAllocThreads),
-                                    args, 0, s);
+                                    args, size_t(kNoAllocThreads) * kSlotBytes, s);
     if (e == cudaErrorCooperativeLaunchTooLarge) {
         cudaGetLastError();
         return fail_c(DPDR_ERR_NOT_COOPERATIVE, "no-alloc: CTAs cannot be co-resident");

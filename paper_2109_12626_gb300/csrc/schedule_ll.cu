@@ -336,7 +336,7 @@ const void* schedule_ll_kernel_for(int dtype)
 int schedule_transport(const Plan* P)
 {
     if (P->sched_transport) return P->sched_transport;
-    const int R = std::max(1, P->sched_ranks_per_cta);
+    const int R = std::max(1, P->sched_rpc_ref);
     const int64_t bytes = int64_t(P->p) * P->m * int64_t(P->esize);
     const int64_t cap = R == 1 ? (P->p >= 1024 ? int64_t(24) << 20 : int64_t(12) << 20)
                       : R == 2 ? int64_t(8) << 20 : 0;
@@ -347,7 +347,7 @@ int schedule_transport(const Plan* P)
 // kBatchWords words for each thread.  The plan sizes column slices by it.
 int64_t schedule_ll_slice_elems(const Plan* P)
 {
-    return int64_t(P->sched_threads) * (kBatchWords / int64_t(P->esize / 4));
+    return int64_t(P->sched_threads_used) * (kBatchWords / int64_t(P->esize / 4));
 }
 
 // Bytes of the word arrays (up and down, p rows of m elements, 8 bytes per
@@ -410,7 +410,7 @@ int schedule_ll_launch(Plan* P, cudaStream_t s)
     a.nchunks = P->sched_chunks;
     void* args[] = {&a};
     cudaError_t e = cudaLaunchCooperativeKernel(schedule_ll_kernel_for(P->dtype),
-                                                dim3(P->sched_ctas), dim3(P->sched_threads),
+                                                dim3(P->sched_ctas), dim3(P->sched_threads_used),
                                                 args, 0, s);
     if (e == cudaErrorCooperativeLaunchTooLarge) {
         cudaGetLastError();

@@ -71,3 +71,16 @@ def test_not_cooperative_is_an_error_not_a_hang(pkg):
         plan.set(pkg.OPT_SCHED_RANKS_PER_CTA, 0)   # fewest that fit: works
         plan.allreduce_schedule(xs, ys)
         plan.sync()
+
+
+def test_wait_limit_is_bounded_above_and_below(pkg):
+    """A wait limit outside [1 us, 10 s] is refused, so no caller can make
+    the schedule kernel's waits unbounded."""
+    from paper_2109_12626_gb300 import DpdrError
+    with pkg.Plan(7, 64, "int32", 4) as plan:
+        for bad in (999, 10_000_000_001, 1 << 62):
+            with pytest.raises(DpdrError) as e:
+                plan.set(pkg.OPT_WAIT_LIMIT_NS, bad)
+            assert e.value.status == pkg.DPDR_ERR_INVALID
+        for good in (1000, 10_000_000_000):
+            plan.set(pkg.OPT_WAIT_LIMIT_NS, good)

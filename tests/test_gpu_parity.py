@@ -473,7 +473,7 @@ def test_schedule_graph_replay(pkg, orc, transport):
 
 def test_default_block_count(pkg):
     """b == 0: one block with flagged words; otherwise the Sec. 1.2 rule at
-    kappa = 46e6 / (p esize), raised to 4 p m esize / L2 blocks."""
+    kappa = 46e6 / (p esize), raised to 2 p m esize / L2 blocks."""
     import math
     l2 = torch.cuda.get_device_properties(0).L2_cache_size
     with pkg.Plan(288, 2500, "int32", 0) as plan:
@@ -482,7 +482,7 @@ def test_default_block_count(pkg):
         with pkg.Plan(p, m, "int32", 0) as plan:
             assert plan.info()["sched_transport"] == 1
             rule = pkg.block_count_rule(p, m, 46e6 / (p * 4))
-            want = max(rule, math.ceil(4 * p * m * 4 / l2))
+            want = max(rule, math.ceil(2 * p * m * 4 / l2))
             assert plan.query()["b"] == want, (p, m)
             plan.set(pkg.OPT_BLOCKS, 0)
             assert plan.query()["b"] == want
