@@ -43,7 +43,6 @@
 #include <mutex>
 
 #include "schedule_common.cuh"
-#include "tma.cuh"
 
 namespace dpdr {
 namespace {
@@ -363,7 +362,7 @@ __device__ __noinline__ void discard_consumed(const SchedArgs& a, const char* ro
     const uintptr_t lo = (reinterpret_cast<uintptr_t>(row + s * Op::kEsize) + 127) & ~uintptr_t(127);
     const uintptr_t hi = reinterpret_cast<uintptr_t>(row + e * Op::kEsize) & ~uintptr_t(127);
     for (uintptr_t l = lo + uintptr_t(grp.tid) * 128; l < hi; l += uintptr_t(grp.size) * 128)
-        tma::discard_l2_line(reinterpret_cast<const void*>(l));
+        asm volatile("discard.global.L2 [%0], 128;" ::"l"(l) : "memory");
 }
 
 __device__ __forceinline__ char* ring_base(const SchedArgs& a, int side, int j, int g,
