@@ -17,6 +17,11 @@
  *   O4  orc_simulate     event-level simulation of Algorithm 1: explicit
  *                        per-processor lists of bidirectional exchanges,
  *                        paired by a rendezvous matcher, unit-step clock
+ *   O5  orc_simulate_rb  event-level simulation of the alternative that
+ *                        Sec. 1.2 analyses and Sec. 2 measures (item 3,
+ *                        "User-Allreduce1"): a pipelined reduction to the
+ *                        root of one binary tree, then a pipelined
+ *                        broadcast from it, the same b blocks in both
  *
  * Element types: int32 sum (wrapping two's complement, computed as uint32),
  * float32 sum (IEEE round-to-nearest-even, no contraction), 2x2 uint32 matrix
@@ -58,7 +63,10 @@ enum {
  * 0 = none. 1 = swap the operands of the child_0 combine in the tree fold.
  * 2 = drop the child_1 term in the tree fold. 3 = use node height instead of
  * depth for d_i in the simulation. 4 = both roots apply t (.) Y in the
- * simulation (ignores the non-commutative rule of Algorithm 1). */
+ * simulation (ignores the non-commutative rule of Algorithm 1).
+ * 5 = in the reduce-then-broadcast simulation the root starts broadcasting
+ * each block as soon as child_0's part of it has arrived, before child_1's
+ * part and before its reduction phase has ended. */
 static int g_mutation = 0;
 void orc_set_mutation(int k) { g_mutation = k; }
 
@@ -563,4 +571,201 @@ int orc_simulate(int p, int64_t m, int b, int dt, const void* x, void* y,
                  int64_t* stats, int* last_round)
 {
     return orc_simulate_topo(p, 0, m, b, dt, x, y, stats, last_round);
+}
+
+/* ------------------------------------------------------------------ O5 ---
+ * Pipelined reduce, then pipelined broadcast, on one binary tree (the
+ * alternative of Sec. 1.2 whose cost is 2(2h + 2(b-1))(alpha + beta m/b),
+ * and the "pipelined reduce followed by a pipelined broadcast with the same
+ * pipeline block size using a single binary tree" of Sec. 2, item 3).  The
+ * tree is the one-tree topology (topo 1): complete, post-order, root p-1.
+ *
+ * Communication model: every processor has one send port and one receive
+ * port (it can send one block and receive another in the same step, as in
+ * the bidirectional model of Sec. 1.2); a transfer of one block takes one
+ * unit step on the sender's send port and the receiver's receive port.
+ * Each port works through a fixed list of transfers in order:
+ *   reduction phase, blocks j = 0..b-1:
+ *     receive port: child_0's partial block j, then child_1's;
+ *                   Y[j] = t (.) Y[j] for each, so Y[j] = v(c1) (.) (v(c0) (.) x_i)
+ *     send port:    Y[j] to the parent, once both children's blocks j arrived
+ *   broadcast phase, blocks j = 0..b-1:
+ *     receive port: final block j from the parent, Y[j] = t
+ *     send port:    Y[j] to child_0, then to child_1, once held
+ * The two phases are two collective operations called one after the other:
+ * a processor takes part in the broadcast only when all its reduction
+ * transfers (on both ports) are done, and the root broadcasts only after it
+ * has reduced all b blocks.  A transfer happens when the sender's next send
+ * and the receiver's next receive name each other (with equal block index
+ * and phase, else ORC_EMISMATCH), at step max(send port free, receive port
+ * free, data ready) + 1.
+ *
+ * x is [p][m]; y ([p][m]) receives every processor's final Y.
+ * stats[0] total steps (largest port clock)
+ * stats[1] step at which the root holds all b reduced blocks
+ * stats[2] number of transfers
+ * stats[3] step at which the last processor holds final block 0
+ * stats[4] largest number of (.) applications on one block at one processor
+ * stats[5] step at which the root's first broadcast transfer starts
+ */
+typedef struct {
+    int partner;
+    int blk;
+    int phase; /* 0 reduction, 1 broadcast */
+} rbop;
+
+int orc_simulate_rb(int p, int64_t m, int b, int dt, const void* x, void* y,
+                    int64_t* stats)
+{
+    size_t s = esize(dt);
+    if (p < 1 || m < 1 || b < 1 || b > m || s == 0) return ORC_EINVAL;
+    int rc = ORC_OK;
+    size_t bytes = (size_t)m * s;
+    char* Y = (char*)y;
+    int* T = (int*)malloc(sizeof(int) * 5 * (size_t)p);
+    rbop** snd = (rbop**)calloc((size_t)p, sizeof(rbop*));
+    rbop** rcv = (rbop**)calloc((size_t)p, sizeof(rbop*));
+    int64_t* nsnd = (int64_t*)calloc((size_t)p, sizeof(int64_t));
+    int64_t* nrcv = (int64_t*)calloc((size_t)p, sizeof(int64_t));
+    int64_t* sp = (int64_t*)calloc((size_t)p, sizeof(int64_t));
+    int64_t* rp = (int64_t*)calloc((size_t)p, sizeof(int64_t));
+    int64_t* sfree = (int64_t*)calloc((size_t)p, sizeof(int64_t));
+    int64_t* rfree = (int64_t*)calloc((size_t)p, sizeof(int64_t));
+    int64_t* red_left = (int64_t*)calloc((size_t)p, sizeof(int64_t)); /* reduction transfers to go */
+    int64_t* red_end = (int64_t*)calloc((size_t)p, sizeof(int64_t));
+    /* per processor and block: children's blocks still to come, the step at
+     * which the block is reduced (-1: not yet), the step at which the final
+     * block is held (-1: not yet) */
+    int* left = (int*)malloc(sizeof(int) * (size_t)p * (size_t)b);
+    int64_t* ready = (int64_t*)malloc(sizeof(int64_t) * (size_t)p * (size_t)b);
+    int64_t* fin = (int64_t*)malloc(sizeof(int64_t) * (size_t)p * (size_t)b);
+    char* early = (char*)malloc(bytes); /* planted mistake 5: the root's early copies */
+    if (!T || !snd || !rcv || !nsnd || !nrcv || !sp || !rp || !sfree || !rfree ||
+        !red_left || !red_end || !left || !ready || !fin || !early) {
+        rc = ORC_ENOMEM;
+        goto done;
+    }
+    int *par = T, *c0 = T + p, *c1 = T + 2 * p, *du = T + 3 * p, *dep = T + 4 * p;
+    rc = orc_trees_topo(p, 1, par, c0, c1, du, dep);
+    if (rc) goto done;
+    memcpy(Y, x, bytes * (size_t)p); /* Y <- x_i */
+    int root = p - 1;
+    int64_t ntransfers = 0, max_ops = 0;
+    for (int i = 0; i < p; i++) {
+        int nch = (c0[i] >= 0) + (c1[i] >= 0);
+        snd[i] = (rbop*)malloc(sizeof(rbop) * (size_t)b * 3);
+        rcv[i] = (rbop*)malloc(sizeof(rbop) * (size_t)b * 3);
+        if (!snd[i] || !rcv[i]) { rc = ORC_ENOMEM; goto done; }
+        int64_t ks = 0, kr = 0;
+        for (int j = 0; j < b; j++) { /* reduction */
+            if (c0[i] >= 0) rcv[i][kr++] = (rbop){c0[i], j, 0};
+            if (c1[i] >= 0) rcv[i][kr++] = (rbop){c1[i], j, 0};
+            if (par[i] >= 0) snd[i][ks++] = (rbop){par[i], j, 0};
+        }
+        red_left[i] = ks + kr;
+        for (int j = 0; j < b; j++) { /* broadcast */
+            if (par[i] >= 0) rcv[i][kr++] = (rbop){par[i], j, 1};
+            if (c0[i] >= 0) snd[i][ks++] = (rbop){c0[i], j, 1};
+            if (c1[i] >= 0) snd[i][ks++] = (rbop){c1[i], j, 1};
+        }
+        nsnd[i] = ks;
+        nrcv[i] = kr;
+        ntransfers += ks;
+        for (int j = 0; j < b; j++) {
+            left[(size_t)i * b + j] = nch;
+            ready[(size_t)i * b + j] = nch ? -1 : 0; /* a leaf's block is x_i */
+            fin[(size_t)i * b + j] = -1;
+        }
+        if (nch > max_ops) max_ops = nch;
+    }
+    int64_t done_tr = 0, first_bcast = -1;
+    while (done_tr < ntransfers) {
+        int progress = 0;
+        for (int a = 0; a < p; a++) {
+            while (sp[a] < nsnd[a]) {
+                rbop* o = &snd[a][sp[a]];
+                int B = o->partner;
+                if (rp[B] >= nrcv[B]) break;
+                rbop* q = &rcv[B][rp[B]];
+                if (q->partner != a) break; /* the receiver expects someone else first */
+                if (q->blk != o->blk || q->phase != o->phase) { rc = ORC_EMISMATCH; goto done; }
+                int j = o->blk;
+                int64_t rdy;
+                const char* src = Y + (size_t)a * bytes;
+                if (o->phase == 0) {
+                    rdy = ready[(size_t)a * b + j];
+                    if (rdy < 0) break;
+                } else {
+                    /* both ends have finished their reduction transfers */
+                    if (red_left[B] > 0) break;
+                    if (a == root && g_mutation == 5) {
+                        /* planted: broadcast once child_0's part has arrived */
+                        rdy = fin[(size_t)a * b + j];
+                        if (rdy < 0) break;
+                        src = early;
+                    } else {
+                        if (red_left[a] > 0) break;
+                        rdy = (a == root) ? ready[(size_t)a * b + j] : fin[(size_t)a * b + j];
+                        if (rdy < 0) break;
+                        if (red_end[a] > rdy) rdy = red_end[a];
+                    }
+                    if (red_end[B] > rdy) rdy = red_end[B];
+                }
+                int64_t t = sfree[a] > rfree[B] ? sfree[a] : rfree[B];
+                if (rdy > t) t = rdy;
+                t += 1;
+                sfree[a] = rfree[B] = t;
+                sp[a]++;
+                rp[B]++;
+                done_tr++;
+                progress = 1;
+                int64_t s0 = blk_start(m, b, j);
+                int64_t len = blk_start(m, b, j + 1) - s0;
+                char* dst = Y + (size_t)B * bytes + (size_t)s0 * s;
+                const char* t_blk = src + (size_t)s0 * s;
+                if (o->phase == 0) {
+                    opv(dt, t_blk, dst, dst, len); /* Y[j] = t (.) Y[j] */
+                    size_t k = (size_t)B * b + j;
+                    if (--left[k] == 0) ready[k] = t;
+                    /* planted mistake 5 keeps the root's block as it is
+                     * after child_0's part */
+                    if (g_mutation == 5 && B == root && a == c0[root]) {
+                        memcpy(early + (size_t)s0 * s, dst, (size_t)len * s);
+                        fin[k] = t;
+                    }
+                    if (--red_left[a] == 0) red_end[a] = t;
+                    if (--red_left[B] == 0) red_end[B] = t;
+                } else {
+                    memcpy(dst, t_blk, (size_t)len * s); /* final block */
+                    fin[(size_t)B * b + j] = t;
+                    if (a == root && (first_bcast < 0 || t - 1 < first_bcast)) first_bcast = t - 1;
+                }
+            }
+        }
+        if (!progress) { rc = ORC_EDEADLOCK; goto done; }
+    }
+    int64_t tot = 0, f0 = 0;
+    for (int i = 0; i < p; i++) {
+        if (sfree[i] > tot) tot = sfree[i];
+        if (rfree[i] > tot) tot = rfree[i];
+        int64_t h0 = (i == root) ? ready[(size_t)i * b] : fin[(size_t)i * b];
+        if (h0 > f0) f0 = h0;
+    }
+    int64_t rend = 0;
+    for (int j = 0; j < b; j++)
+        if (ready[(size_t)root * b + j] > rend) rend = ready[(size_t)root * b + j];
+    stats[0] = tot;
+    stats[1] = rend;
+    stats[2] = ntransfers;
+    stats[3] = f0;
+    stats[4] = max_ops;
+    stats[5] = first_bcast;
+
+done:
+    if (snd) for (int i = 0; i < p; i++) free(snd[i]);
+    if (rcv) for (int i = 0; i < p; i++) free(rcv[i]);
+    free(snd); free(rcv); free(nsnd); free(nrcv); free(sp); free(rp); free(sfree);
+    free(rfree); free(red_left); free(red_end); free(left); free(ready); free(fin);
+    free(early); free(T);
+    return rc;
 }

@@ -13,6 +13,9 @@ Functions and the passages they follow:
   tree_fold(x, dt)         post-order bracketing, Sec. 1.1 + Algorithm 1 roots
   allreduce(x, dt)         tree fold copied to all p rows
   simulate(x, dt, b)       event-level simulation of Algorithm 1
+  simulate_rb(x, dt, b)    event-level simulation of a pipelined reduce, then
+                           a pipelined broadcast, on one tree (Sec. 1.2 cost
+                           analysis; Sec. 2, item 3)
   left_fold_f64(x)         float32 inputs folded in double, with sum |x_i|
 """
 from __future__ import annotations
@@ -73,10 +76,14 @@ def lib():
         L.orc_left_fold_f64.argtypes = [ctypes.c_int, ctypes.c_int64,
                                         ctypes.c_void_p, ctypes.c_void_p,
                                         ctypes.c_void_p]
+        L.orc_simulate_rb.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_int,
+                                      ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p,
+                                      ctypes.POINTER(ctypes.c_int64)]
         L.orc_set_mutation.argtypes = [ctypes.c_int]
         for f in (L.orc_trees, L.orc_left_fold, L.orc_tree_fold,
                   L.orc_allreduce, L.orc_simulate, L.orc_left_fold_f64,
-                  L.orc_trees_topo, L.orc_tree_fold_topo, L.orc_simulate_topo):
+                  L.orc_trees_topo, L.orc_tree_fold_topo, L.orc_simulate_topo,
+                  L.orc_simulate_rb):
             f.restype = ctypes.c_int
         _lib = L
     return _lib
@@ -163,6 +170,19 @@ def simulate(x: np.ndarray, dt: int, b: int, topo: int = DUAL):
                    "max_ops_nonroot", "max_ops_root", "void_skipped"),
                   [int(v) for v in stats]))
     return y, st, last
+
+
+def simulate_rb(x: np.ndarray, dt: int, b: int):
+    """Event-level simulation of the pipelined reduce, then pipelined
+    broadcast, on one tree (Sec. 1.2, Sec. 2 item 3); returns (Y [p][m...],
+    stats)."""
+    x, p, m = _shape(x, dt)
+    y = np.empty_like(x)
+    stats = (ctypes.c_int64 * 6)()
+    _check(lib().orc_simulate_rb(p, m, b, dt, _ptr(x), _ptr(y), stats))
+    st = dict(zip(("steps", "reduce_end_root", "transfers", "first_block_last",
+                   "max_ops", "first_bcast_start"), [int(v) for v in stats]))
+    return y, st
 
 
 def left_fold_f64(x: np.ndarray):
