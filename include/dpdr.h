@@ -252,6 +252,26 @@ int dpdr_allreduce(dpdr_plan_t plan, const void* const* x, void* const* y,
 int dpdr_allreduce_schedule(dpdr_plan_t plan, const void* const* x,
                             void* const* y, dpdr_stream_t stream);
 
+/* The alternative that Sec. 1.2 analyses and Sec. 2 (item 3) measures
+ * against Algorithm 1: a pipelined reduction of the plan's b blocks to the
+ * root of one binary tree, followed by a pipelined broadcast of them from
+ * the root, each phase moving blocks in one direction only.  Needs a plan
+ * made with DPDR_TOPO_SINGLE (the complete post-order tree over all p ranks,
+ * root p-1); any other plan is DPDR_ERR_INVALID.  Runs as one cooperative
+ * persistent launch with the same CTA layout, handshakes, block passes and
+ * bounded waits as dpdr_allreduce_schedule's counters transport: in the
+ * reduction every rank forms Y[j] = v(child_1) (.) (v(child_0) (.) x_i) for
+ * j = 0..b-1 and publishes it to its parent; once its reduction is done it
+ * receives the final blocks from its parent in order and publishes each to
+ * its children (the root publishes all b once its reduction is done).  The
+ * result is the one tree's bracketing, bit for bit the same as
+ * dpdr_allreduce and dpdr_allreduce_schedule on the same plan.  x, y: host
+ * arrays of p device pointers, as for dpdr_allreduce; in place allowed.
+ * Asynchronous on stream; an expired wait is reported by dpdr_plan_sync.
+ * Two calls on one plan that overlap on the GPU race on its scratch. */
+int dpdr_allreduce_reduce_bcast(dpdr_plan_t plan, const void* const* x,
+                                void* const* y, dpdr_stream_t stream);
+
 /* Host buffers end to end: y_host[i] = x_host[0] (.) ... (.) x_host[p-1]
  * for host memory x_host[i], y_host[i] (all four arguments are host arrays
  * of p pointers).  Two paths:

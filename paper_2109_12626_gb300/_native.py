@@ -42,6 +42,7 @@ SIGNATURES = {
     "dpdr_plan_destroy": (None, [_P]),
     "dpdr_allreduce": (ctypes.c_int, [_P, _P, _P, _P]),
     "dpdr_allreduce_schedule": (ctypes.c_int, [_P, _P, _P, _P]),
+    "dpdr_allreduce_reduce_bcast": (ctypes.c_int, [_P, _P, _P, _P]),
     "dpdr_allreduce_host": (ctypes.c_int, [_P, _P, _P, _P, _P, _P]),
     "dpdr_plan_sync": (ctypes.c_int, [_P, _P]),
     "dpdr_allreduce_schedule_noalloc": (ctypes.c_int, [ctypes.c_int, ctypes.c_int64,
@@ -212,6 +213,14 @@ class Plan:
                                              _ptr_array(ys), _stream(stream)),
                "dpdr_allreduce_schedule")
 
+    def allreduce_reduce_bcast(self, xs: Sequence, ys: Sequence, stream=None) -> None:
+        """Pipelined reduce to the root, then pipelined broadcast, on a
+        one-tree plan (Sec. 1.2; Sec. 2 item 3)."""
+        assert len(xs) == self.p and len(ys) == self.p
+        _check(lib().dpdr_allreduce_reduce_bcast(self._h, _ptr_array(xs),
+                                                 _ptr_array(ys), _stream(stream)),
+               "dpdr_allreduce_reduce_bcast")
+
     def allreduce_host(self, xh: Sequence, yh: Sequence, xd: Sequence | None = None,
                        yd: Sequence | None = None, stream=None) -> None:
         """Host buffers in and out (device buffers as staging when the GPU
@@ -249,3 +258,8 @@ class Bound:
         _check(lib().dpdr_allreduce_schedule(self.plan._h, self.X, self.Y,
                                              _stream(stream)),
                "dpdr_allreduce_schedule")
+
+    def allreduce_reduce_bcast(self, stream=None) -> None:
+        _check(lib().dpdr_allreduce_reduce_bcast(self.plan._h, self.X, self.Y,
+                                                 _stream(stream)),
+               "dpdr_allreduce_reduce_bcast")

@@ -1,5 +1,6 @@
 // api.cpp -- argument checks, rank-pointer staging and the run entry points
 // of the C ABI (dpdr_allreduce, dpdr_allreduce_schedule,
+// dpdr_allreduce_reduce_bcast,
 // dpdr_allreduce_host, dpdr_plan_sync).
 #include <algorithm>
 #include <cstdio>
@@ -122,6 +123,20 @@ extern "C" int dpdr_allreduce_schedule(dpdr_plan_t h, const void* const* x,
     int rc = prepare(P, x, reinterpret_cast<const void* const*>(y), s);
     if (rc) return rc;
     return schedule_transport(P) == 2 ? schedule_ll_launch(P, s) : schedule_launch(P, s);
+}
+
+extern "C" int dpdr_allreduce_reduce_bcast(dpdr_plan_t h, const void* const* x,
+                                           void* const* y, dpdr_stream_t stream)
+{
+    Plan* P = reinterpret_cast<Plan*>(h);
+    if (!P) return fail(DPDR_ERR_INVALID, "dpdr_allreduce_reduce_bcast: NULL plan");
+    if (P->topo != DPDR_TOPO_SINGLE)
+        return fail(DPDR_ERR_INVALID,
+                    "dpdr_allreduce_reduce_bcast: needs a plan made with DPDR_TOPO_SINGLE");
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    int rc = prepare(P, x, reinterpret_cast<const void* const*>(y), s);
+    if (rc) return rc;
+    return schedule_launch(P, s, 1);
 }
 
 // Column chunks of about host_chunk bytes of rank data (default 1 GB), each

@@ -186,7 +186,8 @@ int fused_auto_mode(const Plan* P);             // fused.cu
 int fused_split_prepare(Plan* P, bool force, int depth);  // fused.cu
 int fused_tree_prepare(Plan* P);                // fused_tree.cu: both widths
 int fused_tree_index(const Plan* P);            // fused_tree.cu: the device path's width
-int schedule_launch(Plan* P, cudaStream_t s);   // schedule.cu
+int schedule_launch(Plan* P, cudaStream_t s,   // schedule.cu: Algorithm 1 (algo 0)
+                    int algo = 0);              // or reduce, then broadcast (1)
 int schedule_configure(Plan* P);                // schedule.cu
 int schedule_plan_rpc(Plan* P);                 // schedule.cu: ranks per CTA only
 int schedule_transport(const Plan* P);          // schedule_ll.cu: 1 counters, 2 words

@@ -48,6 +48,8 @@ namespace dpdr {
 namespace {
 
 constexpr int kSchedMaxThreads = sched::kMaxThreads;
+constexpr int kAlgoDoubly = 0;       // Algorithm 1 (dpdr_allreduce_schedule)
+constexpr int kAlgoReduceBcast = 1;  // reduce, then broadcast (dpdr_allreduce_reduce_bcast)
 // Words from one handshake counter to the next: each counter has a 128-byte
 // L2 line of its own, so the release stores and polls of different ranks
 // never queue on one line (with 4-byte counters side by side, the 32 ranks
@@ -488,50 +490,163 @@ __global__ void __launch_bounds__(kSchedMaxThreads, 4) schedule_kernel(SchedArgs
     }
 }
 
-template <class Op>
-const void* kernel_ptr(bool grouped)
+// ------------------------------------------------- reduce, then broadcast
+// The alternative the paper's analysis and experiment compare Algorithm 1
+// with (Sec. 1.2, the reduction to the root followed by a broadcast, both
+// pipelined on binary trees; Sec. 2, item 3): on the one-tree plan, every
+// virtual rank first takes part in a pipelined reduction of the b blocks to
+// the root p-1, then in a pipelined broadcast of them from it.  Each phase
+// moves blocks in one direction only.  The same handshakes, block passes and
+// column slices as Algorithm 1's kernel:
+//   reduction, j = 0..b-1: wait for the children's partial blocks j (a
+//     leaf's is its input x_c, published whole at once), form
+//     Y[j] = t1 (.) (t0 (.) x_i) in y_i and publish it to the parent (at the
+//     root Y[j] is final);
+//   broadcast, j = 0..b-1: wait for the parent's final block j, copy it into
+//     y_i and publish it to the children (the root publishes all b blocks
+//     once its reduction is done).
+// A rank group runs its ranks in increasing order in the reduction (every
+// wait is on a child, a lower rank) and in decreasing order in the
+// broadcast (every wait is on the parent, a higher rank); no reduction wait
+// depends on a broadcast, so with all CTAs resident nothing deadlocks.  An
+// inner child's partial block j is consumed once, by its parent, before the
+// root's reduction ends, and overwritten by the final block only after it.
+template <class Op, bool kG>
+__device__ __forceinline__ bool reduce_step(const SchedArgs& a, int i, int j, int g)
 {
+    constexpr int EPV = Op::kEpv;
+    uint32_t* const up = a.up + int64_t(g) * a.p * kCtr;
+    const int c0 = __ldg(a.child0 + i), c1 = __ldg(a.child1 + i);
+    const int par = __ldg(a.parent + i);
+    const char* xi = rank_in(a.x, i);
+    char* yi = rank_out(a.y, i);
+    const int64_t bs = blk_start(a, j), be = blk_start(a, j + 1);
+    const int64_t s = slice_at<EPV>(a, bs, be, g), e = slice_at<EPV>(a, bs, be, g + 1);
+    if (c0 < 0) {
+        if (par >= 0) {
+            // a leaf: its partial blocks are its input, there from the start
+            if (j == 0) publish<kG>(a, up + i * kCtr, uint32_t(a.b), nullptr, 0, i);
+        } else if (xi != yi) {
+            block_pass<Op, kG, 1>(a, yi, xi, nullptr, nullptr, s, e);  // p == 1
+        }
+        return true;
+    }
+    const bool inner0 = __ldg(a.child0 + c0) >= 0;
+    const char* t0 = inner0 ? rank_in(a.y, c0) : rank_in(a.x, c0);
+    const char* t1 = nullptr;
+    bool inner1 = false;
+    Wait w[2];
+    w[0] = Wait{up + c0 * kCtr, uint32_t(j + 1), 0};
+    if (c1 >= 0) {
+        inner1 = __ldg(a.child0 + c1) >= 0;
+        t1 = inner1 ? rank_in(a.y, c1) : rank_in(a.x, c1);
+        w[1] = Wait{up + c1 * kCtr, uint32_t(j + 1), 1};
+    }
+    if (!cta_wait<kG>(a, w, c1 >= 0 ? 2 : 1, i, j)) return false;
+    fold_children<Op, kG>(a, yi, t0, t1, xi, s, e);
+    if (par >= 0)
+        publish<kG>(a, up + i * kCtr, uint32_t(j + 1), nullptr, 0, i);
+    else
+        group_sync<kG>(a);  // the discards below follow every read
+    if (inner0) discard_consumed<Op, kG>(a, t0, s, e);
+    if (inner1) discard_consumed<Op, kG>(a, t1, s, e);
+    return true;
+}
+
+template <class Op, bool kG>
+__device__ __forceinline__ bool bcast_step(const SchedArgs& a, int i, int j, int g)
+{
+    constexpr int EPV = Op::kEpv;
+    uint32_t* const down = a.down + int64_t(g) * a.p * kCtr;
+    const int par = __ldg(a.parent + i);
+    if (par < 0) {  // the root holds every block: all of them go out at once
+        if (j == 0) publish<kG>(a, down + i * kCtr, uint32_t(a.b), nullptr, 0, i);
+        return true;
+    }
+    const Wait wp{down + par * kCtr, uint32_t(j + 1), 3};
+    if (!cta_wait<kG>(a, &wp, 1, i, j)) return false;
+    const int64_t bs = blk_start(a, j), be = blk_start(a, j + 1);
+    block_pass<Op, kG, 1>(a, rank_out(a.y, i), rank_in(a.y, par), nullptr, nullptr,
+                          slice_at<EPV>(a, bs, be, g), slice_at<EPV>(a, bs, be, g + 1));
+    publish<kG>(a, down + i * kCtr, uint32_t(j + 1), nullptr, 0, i);
+    return true;
+}
+
+template <class Op, bool kG>
+__global__ void __launch_bounds__(kSchedMaxThreads, 4) reduce_bcast_kernel(SchedArgs a)
+{
+    const int g = blockIdx.x / a.nchunks, chunk = blockIdx.x % a.nchunks;
+    const int first = __ldg(a.cta_first + chunk);
+    const int last = __ldg(a.cta_first + chunk + 1);
+    int lo = first, hi = last;
+    if (kG) {
+        const int k = int(threadIdx.x) >> a.lg_gsz;
+        if (k >= a.ngroups) return;  // warps left over by the split
+        const int n = last - first;
+        lo = first + n * k / a.ngroups;
+        hi = first + n * (k + 1) / a.ngroups;
+    }
+    for (int j = 0; j < a.b; j++)
+        for (int i = lo; i < hi; i++)
+            if (!reduce_step<Op, kG>(a, i, j, g)) return;
+    for (int j = 0; j < a.b; j++)
+        for (int i = hi - 1; i >= lo; i--)
+            if (!bcast_step<Op, kG>(a, i, j, g)) return;
+}
+
+template <class Op>
+const void* kernel_ptr(bool grouped, int algo)
+{
+    if (algo == kAlgoReduceBcast)
+        return grouped ? reinterpret_cast<const void*>(&reduce_bcast_kernel<Op, true>)
+                       : reinterpret_cast<const void*>(&reduce_bcast_kernel<Op, false>);
     return grouped ? reinterpret_cast<const void*>(&schedule_kernel<Op, true>)
                    : reinterpret_cast<const void*>(&schedule_kernel<Op, false>);
 }
 
-// The kernel for CTAs that own one rank (grouped = false) or several.
-const void* kernel_for(int dtype, bool grouped)
+// The kernel for CTAs that own one rank (grouped = false) or several:
+// Algorithm 1 (algo kAlgoDoubly) or the reduction then broadcast.
+const void* kernel_for(int dtype, bool grouped, int algo = kAlgoDoubly)
 {
     switch (dtype) {
-    case DPDR_INT32: return kernel_ptr<SumI32>(grouped);
-    case DPDR_FLOAT32: return kernel_ptr<SumF32>(grouped);
-    case DPDR_MAT2X2_F32: return kernel_ptr<MatF32>(grouped);
-    default: return kernel_ptr<MatU32>(grouped);
+    case DPDR_INT32: return kernel_ptr<SumI32>(grouped, algo);
+    case DPDR_FLOAT32: return kernel_ptr<SumF32>(grouped, algo);
+    case DPDR_MAT2X2_F32: return kernel_ptr<MatF32>(grouped, algo);
+    default: return kernel_ptr<MatU32>(grouped, algo);
     }
 }
 
-// CTAs of `threads` threads that fit one SM for the counters kernel (the
-// variant for one rank per CTA, or the grouped one) and the flagged-word
-// kernel alike.
-// The counters kernel's dynamic shared memory (the cp.async slots) for
-// CTAs of `threads` threads.  Beyond 48 KB less the kernel's static shared
-// memory (256 threads) the kernel must be granted the size first.
+// The counters kernels' dynamic shared memory (the cp.async slots) for
+// CTAs of `threads` threads.  Beyond 48 KB less the kernels' static shared
+// memory (256 threads) the kernels must be granted the size first.
 cudaError_t sched_smem(int dtype, bool grouped, int threads, size_t* bytes)
 {
     *bytes = size_t(threads) * kSlotBytes;
     if (*bytes + 1024 <= 48 * 1024) return cudaSuccess;
-    return cudaFuncSetAttribute(kernel_for(dtype, grouped), cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                int(*bytes));
+    cudaError_t e = cudaSuccess;
+    for (int algo : {kAlgoDoubly, kAlgoReduceBcast})
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(kernel_for(dtype, grouped, algo),
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, int(*bytes));
+    return e;
 }
 
+// CTAs of `threads` threads that fit one SM for the counters kernels (the
+// variant for one rank per CTA, or the grouped one) and the flagged-word
+// kernel alike.
 cudaError_t sched_occupancy(int dtype, int threads, bool grouped, int* occ)
 {
-    int o[2] = {0, 0};
+    int o[3] = {0, 0, 0};
     size_t smem = 0;
-    cudaError_t e0 = sched_smem(dtype, grouped, threads, &smem);
-    if (e0 != cudaSuccess) return e0;
-    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o[0], kernel_for(dtype, grouped),
-                                                                  threads, smem);
+    cudaError_t e = sched_smem(dtype, grouped, threads, &smem);
+    for (int algo : {kAlgoDoubly, kAlgoReduceBcast})
+        if (e == cudaSuccess)
+            e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o[algo], kernel_for(dtype, grouped, algo),
+                                                              threads, smem);
     if (e == cudaSuccess)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o[1], schedule_ll_kernel_for(dtype),
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o[2], schedule_ll_kernel_for(dtype),
                                                           threads, 0);
-    *occ = std::min(o[0], o[1]);
+    *occ = std::min({o[0], o[1], o[2]});
     return e;
 }
 
@@ -645,7 +760,7 @@ int schedule_configure(Plan* P)
     return schedule_transport(P) == 2 ? schedule_ll_prepare(P) : DPDR_OK;
 }
 
-int schedule_launch(Plan* P, cudaStream_t s)
+int schedule_launch(Plan* P, cudaStream_t s, int algo)
 {
     if (P->m == 0) return DPDR_OK;
     SchedArgs a;
@@ -686,7 +801,7 @@ int schedule_launch(Plan* P, cudaStream_t s)
     e = sched_smem(P->dtype, P->sched_ranks_per_cta > 1, P->sched_threads_used, &smem);
     if (e != cudaSuccess) return cuda_fail(e, "schedule kernel shared memory");
     void* args[] = {&a};
-    e = cudaLaunchCooperativeKernel(kernel_for(P->dtype, P->sched_ranks_per_cta > 1),
+    e = cudaLaunchCooperativeKernel(kernel_for(P->dtype, P->sched_ranks_per_cta > 1, algo),
                                     dim3(P->sched_ctas), dim3(P->sched_threads_used), args, smem, s);
     if (e == cudaErrorCooperativeLaunchTooLarge) {
         cudaGetLastError();

@@ -99,6 +99,24 @@ int main(int argc, char** argv)
         check(dpdr_plan_sync(plan, NULL), "dpdr_plan_sync") ||
         compare(p, m, yh, want, "dpdr_allreduce_host"))
         return 1;
+    /* reduce-then-broadcast needs a one-tree plan */
+    if (dpdr_allreduce_reduce_bcast(plan, (const void* const*)xd, yd, NULL) != DPDR_ERR_INVALID) {
+        printf("dpdr_allreduce_reduce_bcast accepted a dual-tree plan\n");
+        return 1;
+    }
+    dpdr_plan_destroy(plan);
+
+    /* pipelined reduce, then pipelined broadcast, on one tree */
+    plan = dpdr_plan_topo(p, m, DPDR_INT32, DPDR_OP_SUM, 0, DPDR_TOPO_SINGLE);
+    if (!plan) return check(dpdr_last_error(), "dpdr_plan_topo");
+    for (int i = 0; i < p; i++) cudaMemset(yd[i], 0xff, bytes);
+    if (check(dpdr_allreduce_reduce_bcast(plan, (const void* const*)xd, yd, NULL),
+              "dpdr_allreduce_reduce_bcast") ||
+        check(dpdr_plan_sync(plan, NULL), "dpdr_plan_sync"))
+        return 1;
+    for (int i = 0; i < p; i++)
+        if (cudaMemcpy(yh[i], yd[i], bytes, cudaMemcpyDeviceToHost) != cudaSuccess) return 1;
+    if (compare(p, m, yh, want, "dpdr_allreduce_reduce_bcast")) return 1;
     dpdr_plan_destroy(plan);
 
     /* the allocation-free entry point: no plan at all */
