@@ -55,7 +55,8 @@ KERNEL_SOURCES = {"stream": ("fused_stream.cu", "fused_common.cuh"),
                   "bulk": ("fused_bulk.cu", "fused_common.cuh"),
                   "tree": ("fused_tree.cu", "fused_common.cuh"),
                   "schedule": ("schedule.cu", "schedule_common.cuh"),
-                  "schedule_words": ("schedule_ll.cu", "schedule_common.cuh")}
+                  "schedule_words": ("schedule_ll.cu", "schedule_common.cuh"),
+                  "reduce_bcast": ("schedule.cu", "schedule_common.cuh")}
 LAYOUTS = {1: "stream", 2: "tile", 3: "split", 4: "bulk", 5: "tree"}
 
 
@@ -481,6 +482,8 @@ def run_sweep(args, w) -> int:
             del xs, ys
             torch.cuda.empty_cache()
         return 0
+    if args.sweep == "rb":
+        return run_sweep_rb(args, w)
     # --sweep b
     m = w["m"]
     xs = gen_device_inputs(w, dev)
@@ -514,6 +517,54 @@ def run_sweep(args, w) -> int:
     return 0
 
 
+def run_sweep_rb(args, w) -> int:
+    """--sweep rb: the doubly pipelined dual-root schedule (Algorithm 1)
+    against a pipelined reduce to the root of one tree followed by a
+    pipelined broadcast (the comparison of Sec. 1.2 and Sec. 2, items 3
+    and 4), both with the same pipeline blocks: b = ceil(m / --block-size),
+    or the dual plan's default b.  Also Algorithm 1 on the one tree.  Each
+    time is the min and mean of CUDA-graph replays of one call (launch
+    included).  One JSON line per m."""
+    import torch
+    import paper_2109_12626_gb300 as pkg
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    p, kind, es = w["p"], w["kind"], ESIZE[w["kind"]]
+    top = int(args.m or (1 << 23)).bit_length() - 1
+    ms = ([int(v) for v in args.mlist.split(",")] if args.mlist
+          else [1 << k for k in range(0, top + 1)])
+    for m in ms:
+        ww = dict(w, m=m)
+        xs = gen_device_inputs(ww, dev)
+        ys = [torch.empty_like(x) for x in xs]
+        b = -(-m // args.block_size) if args.block_size else 0
+        rec = {"sweep": "rb", "workload": args.workload, "p": p, "m": m}
+        reps = 5 if p * m >= (1 << 26) else 20
+        with pkg.Plan(p, m, kind, b) as dual:
+            dual.set(pkg.OPT_SCHED_TRANSPORT, 1)
+            b = dual.query()["b"]
+            bd = dual.bind(xs, ys)
+            rec["dual_alg1"] = _stats(_timed_reps(lambda: bd.allreduce_schedule(), reps))
+            dual.sync()
+        with pkg.Plan(p, m, kind, b, topology="single") as one:
+            one.set(pkg.OPT_SCHED_TRANSPORT, 1)
+            bo = one.bind(xs, ys)
+            rec["single_alg1"] = _stats(_timed_reps(lambda: bo.allreduce_schedule(), reps))
+            rec["single_reduce_bcast"] = _stats(_timed_reps(lambda: bo.allreduce_reduce_bcast(),
+                                                            reps))
+            one.sync()
+        rec["b"] = b
+        rec["ratio_rb_over_dual"] = round(rec["single_reduce_bcast"]["us_min"]
+                                          / rec["dual_alg1"]["us_min"], 3)
+        rec["ratio_rb_over_single"] = round(rec["single_reduce_bcast"]["us_min"]
+                                            / rec["single_alg1"]["us_min"], 3)
+        rec["dual_gbs"] = round(2 * p * m * es / (rec["dual_alg1"]["us_min"] * 1e-6) / 1e9, 2)
+        print(json.dumps(rec), flush=True)
+        del xs, ys
+        torch.cuda.empty_cache()
+    return 0
+
+
 # ---------------------------------------------------------------- main
 def main(argv=None) -> int:
     ap = argparse.ArgumentParser()
@@ -522,7 +573,8 @@ def main(argv=None) -> int:
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--m", type=int, default=None, help="override m (sweeps)")
-    ap.add_argument("--kernel", choices=("fused", "schedule"), default="fused")
+    ap.add_argument("--kernel", choices=("fused", "schedule", "reduce_bcast"), default="fused",
+                    help="reduce_bcast: pipelined reduce then broadcast on one tree")
     ap.add_argument("--b", type=int, default=None, help="pipeline blocks (schedule)")
     ap.add_argument("--mode", type=int, default=0,
                     help="fused layout: 0 auto, 1 stream, 2 tile, 3 split, 4 bulk, 5 tree")
@@ -531,7 +583,7 @@ def main(argv=None) -> int:
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
-    ap.add_argument("--sweep", choices=("m", "b"), default=None,
+    ap.add_argument("--sweep", choices=("m", "b", "rb"), default=None,
                     help="m: all m = 2^k up to --m; b: schedule time against b")
     ap.add_argument("--blist", default="1,2,4,8,16,32,64,128,256,512,1024")
     ap.add_argument("--topology", choices=("dual", "single"), default="dual",
@@ -548,6 +600,8 @@ def main(argv=None) -> int:
                     help="time the oracle's event-level simulation of Algorithm 1 (CPU)")
     args = ap.parse_args(argv)
     args.warmup = max(args.warmup, 3)
+    if args.kernel == "reduce_bcast":
+        args.topology = "single"   # the variant runs on the one-tree plan
 
     world, rank, local = dist_env()
     w = workload(args.workload, args.m)
@@ -590,7 +644,8 @@ def main(argv=None) -> int:
     if args.mode:
         plan.set(pkg.OPT_FUSED_MODE, args.mode)
     stream = torch.cuda.current_stream(dev)
-    run = plan.allreduce if args.kernel == "fused" else plan.allreduce_schedule
+    run = {"fused": plan.allreduce, "schedule": plan.allreduce_schedule,
+           "reduce_bcast": plan.allreduce_reduce_bcast}[args.kernel]
     algo_bytes = 2 * p * m * es
 
     for _ in range(args.warmup):
@@ -603,7 +658,8 @@ def main(argv=None) -> int:
           for _ in range(args.steps)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     bound = plan.bind(xs, ys)
-    go = bound.allreduce if args.kernel == "fused" else bound.allreduce_schedule
+    go = {"fused": bound.allreduce, "schedule": bound.allreduce_schedule,
+          "reduce_bcast": bound.allreduce_reduce_bcast}[args.kernel]
     # inputs that L2 could hold: write a buffer of twice L2 before every step
     # and time the steps by their own events, so each step starts cold
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
@@ -682,6 +738,7 @@ def main(argv=None) -> int:
 
     info = plan.info()
     layout = (LAYOUTS[args.mode or info["auto_mode"]] if args.kernel == "fused"
+              else "reduce_bcast" if args.kernel == "reduce_bcast"
               else ("schedule", "schedule_words")[info["sched_transport"] - 1])
     launches_per_step = 2 if layout == "split" else 1
     line = {
