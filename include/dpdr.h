@@ -310,9 +310,13 @@ int dpdr_plan_sync(dpdr_plan_t plan, dpdr_stream_t stream);
  * other allocating routine.
  *
  * It runs the same schedule kernel as dpdr_allreduce_schedule, with the same
- * result, using a scratch array of DPDR_NOALLOC_SCRATCH_BYTES that is
- * statically reserved in device memory on every GPU that loads the library
- * and held until the process exits.  That array holds the rank-pointer and
+ * result, using a scratch array of DPDR_NOALLOC_SCRATCH_BYTES in device
+ * memory.  The array is created when the library's device code is loaded on
+ * a GPU, and held until the process exits.  With CUDA's default lazy module
+ * loading that happens at the first call into this library on that device,
+ * so a caller that must not allocate during some section makes one call
+ * first (any dpdr call on that device, this one included) or sets
+ * CUDA_MODULE_LOADING=EAGER.  That array holds the rank-pointer and
  * tree tables, the handshake counters, the error word and the dual roots'
  * exchange slots (4 slots of one pipeline block each).  Limits: p <=
  * DPDR_NOALLOC_MAX_RANKS, and the tables plus 4 slots of ceil(m/b) elements
@@ -326,7 +330,9 @@ int dpdr_plan_sync(dpdr_plan_t plan, dpdr_stream_t stream);
  * The call is synchronous: it returns after stream has finished the
  * kernel, with DPDR_ERR_TIMEOUT if one of its bounded waits expired.  The
  * first call on each device looks up the array's device address (with that
- * device current) and keeps it.  Every call shares the one array and
+ * device current) and keeps it; make that first call before any stream
+ * capture.  The kept address does not survive cudaDeviceReset: after a
+ * reset, do not call this entry point again in the process.  Every call shares the one array and
  * re-initialises what must start at zero; calls that overlap on the GPU
  * (from two host threads, or on two streams) race and must not be made. */
 #define DPDR_NOALLOC_SCRATCH_BYTES (8u << 20)

@@ -5,17 +5,21 @@ It is for callers that cannot allocate device memory on the call path
 stall the device mid-run): it needs no plan and keeps its scratch in a
 statically reserved device array.  These tests call it through the C ABI
 and check, on two calls in a row with different inputs (the shared scratch
-keeps the previous call's contents), that its outputs equal those of the
-plan-based dpdr_allreduce_schedule bit for bit -- the same tolerance every
-parity test here uses -- and that sizes beyond its stated limits are
-refused with an error instead of being run."""
+keeps the previous call's contents), that its outputs equal the CPU
+oracle's tree fold bit for bit -- the same tolerance every parity test here
+uses -- and those of the plan-based dpdr_allreduce_schedule; that sizes
+beyond its stated limits are refused with an error instead of being run;
+and that a large block the scratch admits gives the right result.  The
+entry point builds the trees on the device itself, so the cases include
+p = 1 (one rank, no tree) and p = 2^k - 1, 2^k, 2^k + 1 (the shapes where a
+complete tree's last level is full, has one node, or has one missing)."""
 import ctypes
 
 import numpy as np
 import pytest
 import torch
 
-from gpu_util import bits, empty_like_ranks, host_inputs, to_device
+from gpu_util import bits, empty_like_ranks, expect_bits, host_inputs, to_device
 
 pytestmark = pytest.mark.gpu
 
@@ -37,14 +41,21 @@ def _call_noalloc(N, p, m, dt, op, b, xs, ys):
     return L.dpdr_allreduce_schedule_noalloc(p, m, dt, op, b, X, Y, stream)
 
 
+def _want(orc, x, kind):
+    dt = {"int32": orc.I32, "float32": orc.F32, "mat2x2u32": orc.MAT}[kind]
+    return expect_bits(orc.tree_fold(x, dt))
+
+
 # p = 3000 puts several ranks on each CTA (rank groups)
 CASES = [("int32", 7, 1000, 4), ("mat2x2u32", 36, 4099, 16),
          ("float32", 1152, 4099, 0), ("float32", 32, 65541, 64), ("int32", 2, 3, 3),
-         ("int32", 3000, 257, 2)]
+         ("int32", 3000, 257, 2), ("float32", 1, 100, 3), ("float32", 63, 999, 5),
+         ("int32", 64, 1001, 7), ("float32", 65, 1003, 4), ("int32", 127, 500, 2),
+         ("float32", 255, 257, 1), ("int32", 257, 300, 3)]
 
 
 @pytest.mark.parametrize("kind,p,m,b", CASES)
-def test_noalloc_matches_planned_schedule_twice(native, kind, p, m, b):
+def test_noalloc_matches_oracle_and_planned_schedule_twice(native, orc, kind, p, m, b):
     import paper_2109_12626_gb300 as pkg
     N = native
     dt = N.DTYPES[kind]
@@ -52,6 +63,7 @@ def test_noalloc_matches_planned_schedule_twice(native, kind, p, m, b):
     dev = torch.device("cuda:0")
     for seed in (51, 52):                     # two calls in a row
         x = host_inputs(kind, seed, p, m)
+        want = _want(orc, x, kind)
         xs, _ = to_device(x, kind, dev)
         ref, _ = empty_like_ranks(xs, fill=-1)
         with pkg.Plan(p, m, kind, b) as plan:
@@ -61,10 +73,11 @@ def test_noalloc_matches_planned_schedule_twice(native, kind, p, m, b):
         rc = _call_noalloc(N, p, m, dt, op, b, xs, got)
         assert rc == N.DPDR_OK, N.lib().dpdr_last_error_message()
         for i in range(p):
+            assert np.array_equal(bits(got[i]), want), (seed, i)
             assert np.array_equal(bits(got[i]), bits(ref[i])), (seed, i)
 
 
-def test_noalloc_refuses_sizes_beyond_its_limits(native):
+def test_noalloc_refuses_sizes_beyond_its_limits(native, orc):
     N = native
     dev = torch.device("cuda:0")
     L = N.lib()
@@ -81,6 +94,12 @@ def test_noalloc_refuses_sizes_beyond_its_limits(native):
     rc = _call_noalloc(N, p, m, N.DPDR_INT32, N.DPDR_OP_SUM, 1, xs, ys)
     assert rc == N.DPDR_ERR_INVALID
     assert b"larger b" in L.dpdr_last_error_message()
-    # the same size with enough blocks runs
+    # the same size with enough blocks runs, and is right
+    x = host_inputs("int32", 53, p, m)
+    want = _want(orc, x, "int32")
+    xs, _ = to_device(x, "int32", dev)
+    ys, _ = empty_like_ranks(xs, fill=-5)
     rc = _call_noalloc(N, p, m, N.DPDR_INT32, N.DPDR_OP_SUM, 64, xs, ys)
-    assert rc == N.DPDR_OK
+    assert rc == N.DPDR_OK, L.dpdr_last_error_message()
+    for y in ys:
+        assert np.array_equal(bits(y), want)
