@@ -381,6 +381,16 @@ def fit_cost_model(p: int, m: int, points, topology: str = "dual"):
     return float(coef[0]), float(coef[1]), float(coef[2])
 
 
+def set_schedule_options(pkg, plan, args) -> None:
+    """The schedule kernels' transport, CTA layout, threads and slices."""
+    plan.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[args.transport])
+    if args.sched_threads:
+        plan.set(pkg.OPT_SCHED_THREADS, args.sched_threads)
+    plan.set(pkg.OPT_SCHED_LAYOUT, args.sched_layout)
+    if args.sched_slices:
+        plan.set(pkg.OPT_SCHED_SLICES, args.sched_slices)
+
+
 def _timed(fn, reps, stream, graph=False):
     import torch
     for _ in range(2):
@@ -460,7 +470,7 @@ def run_sweep(args, w) -> int:
                    "topology": args.topology}
             b0 = -(-m // args.block_size) if args.block_size else 0
             with pkg.Plan(p, m, kind, b0, topology=args.topology) as plan:
-                plan.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[args.transport])
+                set_schedule_options(pkg, plan, args)
                 if args.mode:
                     plan.set(pkg.OPT_FUSED_MODE, args.mode)
                 bd = plan.bind(xs, ys)
@@ -476,6 +486,7 @@ def run_sweep(args, w) -> int:
                 rec["schedule"] = dict(st, b=info["b"],
                                        gbs=round(2 * p * m * es / (st["us"] * 1e-6) / 1e9, 2),
                                        slices=plan.info()["sched_slices"],
+                                       sched_layout=plan.info()["sched_layout"],
                                        transport=("counters", "words")[
                                            info["sched_transport"] - 1])
             print(json.dumps(rec), flush=True)
@@ -492,7 +503,7 @@ def run_sweep(args, w) -> int:
     points = []
     for b in bs:
         with pkg.Plan(p, m, kind, b, topology=args.topology) as plan:
-            plan.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[args.transport])
+            set_schedule_options(pkg, plan, args)
             bd = plan.bind(xs, ys)
             t = _timed(lambda: bd.allreduce_schedule(), 5 if m >= (1 << 20) else 10, None,
                        graph=True)
@@ -542,12 +553,14 @@ def run_sweep_rb(args, w) -> int:
         reps = 5 if p * m >= (1 << 26) else 20
         with pkg.Plan(p, m, kind, b) as dual:
             dual.set(pkg.OPT_SCHED_TRANSPORT, 1)
+            dual.set(pkg.OPT_SCHED_LAYOUT, args.sched_layout)
             b = dual.query()["b"]
             bd = dual.bind(xs, ys)
             rec["dual_alg1"] = _stats(_timed_reps(lambda: bd.allreduce_schedule(), reps))
             dual.sync()
         with pkg.Plan(p, m, kind, b, topology="single") as one:
             one.set(pkg.OPT_SCHED_TRANSPORT, 1)
+            one.set(pkg.OPT_SCHED_LAYOUT, args.sched_layout)
             bo = one.bind(xs, ys)
             rec["single_alg1"] = _stats(_timed_reps(lambda: bo.allreduce_schedule(), reps))
             rec["single_reduce_bcast"] = _stats(_timed_reps(lambda: bo.allreduce_reduce_bcast(),
@@ -594,6 +607,12 @@ def main(argv=None) -> int:
     ap.add_argument("--mlist", default=None, help="comma-separated m values for --sweep m")
     ap.add_argument("--host-path", type=int, default=0,
                     help="e2e leg: 0 direct when possible, 1 copy pipeline, 2 direct")
+    ap.add_argument("--sched-layout", type=int, default=0, choices=(0, 1, 2),
+                    help="schedule kernels' CTA layout: 0 auto, 1 rank ranges, 2 by work")
+    ap.add_argument("--sched-threads", type=int, default=0,
+                    help="threads per schedule CTA (0 = automatic)")
+    ap.add_argument("--sched-slices", type=int, default=0,
+                    help="column slices per rank of the schedule kernels (0 = automatic)")
     ap.add_argument("--transport", choices=tuple(TRANSPORTS), default="auto",
                     help="schedule kernel: how blocks pass between virtual ranks")
     ap.add_argument("--oracle-sim", action="store_true",
@@ -638,7 +657,7 @@ def main(argv=None) -> int:
     xs = gen_device_inputs(w, dev)
     ys = [torch.empty_like(x) for x in xs]
     plan = pkg.Plan(p, m, kind, b, topology=args.topology)
-    plan.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[args.transport])
+    set_schedule_options(pkg, plan, args)
     if args.split_depth is not None:
         plan.set(pkg.OPT_SPLIT_DEPTH, args.split_depth)
     if args.mode:
@@ -750,6 +769,8 @@ def main(argv=None) -> int:
         "config": {"workload": args.workload, "p": p, "m": m, "kind": kind,
                    "topology": args.topology,
                    "kernel": args.kernel, "b": info["b"],
+                   "sched_layout": (None if args.kernel == "fused" else
+                                    {1: "rank ranges", 2: "by work"}[info["sched_layout"]]),
                    "fused_mode": args.mode or info["auto_mode"],
                    "split_depth": info["split_depth"] if (args.mode or info["auto_mode"]) == 3 else None,
                    "bytes_per_step": algo_bytes,

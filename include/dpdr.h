@@ -164,8 +164,9 @@ int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
  *                             its partners' waits expire (-1 = off)
  *   DPDR_OPT_SCHED_THREADS    threads per CTA of the schedule kernel
  *                             (64..256, multiple of 32); 0 (default) is
- *                             automatic: 64 with the counters transport,
- *                             128 with flagged words
+ *                             automatic: 128 with the counters transport
+ *                             laid out by work and with flagged words, 64
+ *                             with the counters transport on rank ranges
  *   DPDR_OPT_SCHED_RANKS_PER_CTA  virtual ranks per CTA (0 = fewest that
  *                             fit co-resident)
  *   DPDR_OPT_BLOCKS           change b (same rules as dpdr_plan's b)
@@ -192,7 +193,18 @@ int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
  *                             device; 0 (default) chooses 2 while the p
  *                             inputs total at most 12 MiB (24 MiB from
  *                             p = 1024) with one rank per schedule CTA,
- *                             8 MiB with two, never with more; else 1 */
+ *                             8 MiB with two, never with more; else 1
+ *   DPDR_OPT_SCHED_LAYOUT     how the counters transport of the schedule
+ *                             kernels lays out virtual ranks on CTAs:
+ *                             1 rank ranges -- each CTA owns a contiguous
+ *                             range of ranks; 2 by work -- each rank has
+ *                             warps of its own in proportion to its block
+ *                             passes per round (a leaf one quarter of a
+ *                             CTA, an inner node three quarters, a root a
+ *                             whole CTA), DPDR_ERR_INVALID when one column
+ *                             slice of it does not fit the GPU at once;
+ *                             0 (default) takes 2 where it fits, else 1.
+ *                             Set ranks per CTA always take rank ranges */
 enum {
     DPDR_OPT_FUSED_MODE = 1,
     DPDR_OPT_WAIT_LIMIT_NS = 2,
@@ -204,7 +216,8 @@ enum {
     DPDR_OPT_SCHED_SLICES = 8,
     DPDR_OPT_HOST_CHUNK_BYTES = 9,
     DPDR_OPT_HOST_PATH = 10,
-    DPDR_OPT_SCHED_TRANSPORT = 11
+    DPDR_OPT_SCHED_TRANSPORT = 11,
+    DPDR_OPT_SCHED_LAYOUT = 12
 };
 int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
 
@@ -221,7 +234,9 @@ int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
  *   [15] transport of dpdr_allreduce_schedule: 1 counters, 2 flagged words
  *   [16] 16-byte column units per CTA of the hierarchical tile layout on
  *        device buffers (8 while those CTAs fit in one wave of resident
- *        CTAs, 2 per SM; else 16; host buffers always take 8) */
+ *        CTAs, 2 per SM; else 16; host buffers always take 8)
+ *   [17] CTA layout of the schedule kernels: 1 rank ranges, 2 by work
+ *        (DPDR_OPT_SCHED_LAYOUT; flagged words always take rank ranges) */
 int dpdr_plan_info(dpdr_plan_t plan, int64_t* info, int n);
 
 /* Releases the plan's device and host memory.  The caller must first make

@@ -18,7 +18,8 @@ DPDR_OP_SUM, DPDR_OP_MATMUL = 0, 1
  DPDR_ERR_NOT_COOPERATIVE, DPDR_ERR_OOM) = range(6)
 (OPT_FUSED_MODE, OPT_WAIT_LIMIT_NS, OPT_SKIP_RANK, OPT_SCHED_THREADS,
  OPT_SCHED_RANKS_PER_CTA, OPT_BLOCKS, OPT_SPLIT_DEPTH, OPT_SCHED_SLICES,
- OPT_HOST_CHUNK_BYTES, OPT_HOST_PATH, OPT_SCHED_TRANSPORT) = range(1, 12)
+ OPT_HOST_CHUNK_BYTES, OPT_HOST_PATH, OPT_SCHED_TRANSPORT,
+ OPT_SCHED_LAYOUT) = range(1, 13)
 
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libdpdr.so")
 
@@ -143,7 +144,8 @@ DTYPES = {"int32": DPDR_INT32, "float32": DPDR_FLOAT32,
 INFO_KEYS = ("p", "m", "b", "max_depth", "auto_mode", "sched_ctas",
              "sched_ranks_per_cta", "scratch_bytes", "vector_path",
              "split_depth", "split_subtrees", "split_group", "sched_slices",
-             "topology", "host_path", "sched_transport", "tree_width")
+             "topology", "host_path", "sched_transport", "tree_width",
+             "sched_layout")
 
 
 class Plan:

@@ -86,6 +86,7 @@ struct Plan {
     int sched_slices = 0;      // CTAs per rank (column slices), 0 = auto
     int split_depth = -1;      // cut depth of the split layout, -1 = auto
     int sched_transport = 0;   // schedule kernel: 0 auto, 1 counters, 2 flagged words
+    int sched_layout = 0;      // counters kernels' CTA layout: 0 auto, 1 rank ranges, 2 by work
     int64_t host_chunk = int64_t(1) << 30;  // bytes of rank data per host-pipeline chunk
     int host_path = 0;         // dpdr_allreduce_host: 0 auto, 1 copy pipeline, 2 direct
     int last_host_path = 0;    // path the last dpdr_allreduce_host took (1 or 2)
@@ -103,8 +104,10 @@ struct Plan {
     uint32_t* d_err = nullptr;       // 4 words: status, rank, round, step
     char* d_ring = nullptr;          // dual-root exchange slots: [2][2][slot]
     size_t ring_slot_bytes = 0;
-    int* d_cta_first = nullptr;      // schedule chunk -> first rank (+1 entry)
-    char* d_sched = nullptr;         // own allocation: counters + chunk table
+    int* d_cta_first = nullptr;      // flagged words: chunk -> first rank (+1 entry)
+    int4* d_groups = nullptr;        // counters: [chunks][4] group descriptors
+    int* d_rank_list = nullptr;      // counters: the groups' ranks
+    char* d_sched = nullptr;         // own allocation: counters + CTA tables
     size_t d_sched_bytes = 0;
     // low-latency transport of the schedule kernel (schedule_ll.cu): control
     // words, then the up and down word arrays; own allocation
@@ -159,6 +162,8 @@ struct Plan {
     int sched_rpc_ref = 1;         // ranks per CTA at 128 threads (transport choice)
     int sched_threads_used = 128;  // threads per CTA of the kernel that runs
     int sched_slices_used = 1, sched_chunks = 1;
+    int sched_layout_used = 1;     // 1 rank ranges, 2 by work
+    int sched_slot_bytes = 192;    // counters kernels: shared memory per thread
 };
 
 // host-side builders (plan.cpp)

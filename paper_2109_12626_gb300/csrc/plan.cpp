@@ -454,6 +454,17 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
         if (v < 0 || v > P->p) return fail(DPDR_ERR_INVALID, "ranks per CTA out of range");
         P->sched_rpc = int(v);
         return schedule_configure(P);
+    case DPDR_OPT_SCHED_LAYOUT: {
+        if (v < 0 || v > 2) return fail(DPDR_ERR_INVALID, "schedule layout: 0, 1 or 2");
+        const int was = P->sched_layout;
+        P->sched_layout = int(v);
+        const int rc = schedule_configure(P);
+        if (rc) {
+            P->sched_layout = was;
+            schedule_configure(P);
+        }
+        return rc;
+    }
     case DPDR_OPT_SCHED_SLICES:
         if (v < 0 || v > kMaxSlices) return fail(DPDR_ERR_INVALID, "slices: 0..1024");
         P->sched_slices = int(v);
@@ -512,7 +523,8 @@ extern "C" int dpdr_plan_info(dpdr_plan_t h, int64_t* info, int n)
                                  P->d_ll_bytes + P->tree[0].bytes + P->tree[1].bytes),
                          P->last_vector_path, P->split_s, P->split_nseg, P->split_group,
                          P->sched_slices_used, P->topo, P->last_host_path,
-                         schedule_transport(P), P->tree[fused_tree_index(P)].width};
+                         schedule_transport(P), P->tree[fused_tree_index(P)].width,
+                         P->sched_layout_used};
     const int k = int(sizeof v / sizeof v[0]);
     for (int i = 0; i < n; i++) info[i] = i < k ? v[i] : 0;
     return DPDR_OK;

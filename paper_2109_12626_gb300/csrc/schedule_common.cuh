@@ -20,16 +20,6 @@ inline int group_count(int R, int threads)
     return R < 1 ? 1 : (R < warps ? (R < kMaxGroups ? R : kMaxGroups)
                                   : (warps < kMaxGroups ? warps : kMaxGroups));
 }
-// log2 of the group size: the largest power of two of whole warps that
-// fits threads / groups
-inline int group_lg(int R, int threads)
-{
-    const int per = threads / group_count(R, threads);
-    int lg = 5;
-    while ((64 << (lg - 5)) <= per) lg++;
-    return lg;
-}
-
 __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p)
 {
     uint32_t v;
@@ -39,6 +29,10 @@ __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p)
 __device__ __forceinline__ void st_release(uint32_t* p, uint32_t v)
 {
     asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ void st_relaxed(uint32_t* p, uint32_t v)
+{
+    asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 __device__ __forceinline__ uint32_t ld_relaxed(const uint32_t* p)
 {

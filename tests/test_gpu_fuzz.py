@@ -2,8 +2,8 @@
 
 Each case draws, from its own seeded generator, the rank count p (1 to
 3000), m, the block count b, the element type, the topology, the fused
-layout, the schedule kernel's transport, column slices and ranks per CTA,
-and the buffer layout (separate, in place, or only 4-byte aligned), then
+layout, the schedule kernel's transport, CTA layout, column slices and ranks
+per CTA, and the buffer layout (separate, in place, or only 4-byte aligned), then
 checks every output of both kernels bit for bit against the oracle's fold.
 The draws reach combinations no hand-written case names -- blocks of two
 lengths cut into slices, ragged tails under every layout, deep trees with
@@ -39,11 +39,15 @@ def draw(k: int) -> dict:
     ctas = -(-p // max(rpc, 1)) * max(slices, 1) if rpc else 0
     if ctas > 1000:
         rpc = 0
-    return dict(kind=kind, p=p, m=m, b=int(rng.integers(1, min(m, 400) + 1)),
-                topology="single" if rng.random() < 0.25 else "dual",
-                mode=int(rng.integers(0, 6)), transport=int(rng.integers(0, 3)),
-                slices=slices, rpc=rpc,
-                layout=("aligned", "aligned", "in_place", "four_byte")[int(rng.integers(4))])
+    c = dict(kind=kind, p=p, m=m, b=int(rng.integers(1, min(m, 400) + 1)),
+             topology="single" if rng.random() < 0.25 else "dual",
+             mode=int(rng.integers(0, 6)), transport=int(rng.integers(0, 3)),
+             slices=slices, rpc=rpc,
+             layout=("aligned", "aligned", "in_place", "four_byte")[int(rng.integers(4))])
+    # the schedule kernels' CTA layout: automatic (by work where it fits) or
+    # rank ranges, drawn last so the draws above stay as they were
+    c["sched_layout"] = 1 if rng.random() < 0.3 else 0
+    return c
 
 
 @pytest.fixture(scope="module")
@@ -91,6 +95,7 @@ def test_random_configuration(pkg, orc, k):
                 plan.allreduce(xs, ys)
             else:
                 plan.set(pkg.OPT_SCHED_TRANSPORT, c["transport"])
+                plan.set(pkg.OPT_SCHED_LAYOUT, c["sched_layout"])
                 if c["slices"]:
                     plan.set(pkg.OPT_SCHED_SLICES, c["slices"])
                 if c["rpc"]:
@@ -121,9 +126,11 @@ def draw_large(k: int) -> dict:
     # half the cases with blocks of at least 4096 elements (several column
     # slices per rank under the automatic layout)
     bmax = min(m, 2000) if rng.random() < 0.5 else max(1, m // 4096)
-    return dict(kind=kind, p=p, m=m, b=int(rng.integers(1, bmax + 1)),
-                mode=int(rng.integers(0, 6)), transport=int(rng.choice([0, 1, 1, 2])),
-                slices=int(rng.integers(1, 33)) if rng.random() < 0.5 else 0)
+    c = dict(kind=kind, p=p, m=m, b=int(rng.integers(1, bmax + 1)),
+             mode=int(rng.integers(0, 6)), transport=int(rng.choice([0, 1, 1, 2])),
+             slices=int(rng.integers(1, 33)) if rng.random() < 0.5 else 0)
+    c["sched_layout"] = 1 if rng.random() < 0.3 else 0  # drawn last, as above
+    return c
 
 
 def _numpy_inputs(kind, rng, p, m):
@@ -159,6 +166,7 @@ def test_random_large_configuration(pkg, orc, k):
                 plan.allreduce(xs, list(yt.unbind(0)))
             else:
                 plan.set(pkg.OPT_SCHED_TRANSPORT, c["transport"])
+                plan.set(pkg.OPT_SCHED_LAYOUT, c["sched_layout"])
                 if c["slices"]:
                     plan.set(pkg.OPT_SCHED_SLICES, c["slices"])
                 plan.allreduce_schedule(xs, list(yt.unbind(0)))

@@ -93,12 +93,16 @@ def test_fused_matches_oracle(pkg, orc, case, mode):
 
 
 TRANSPORTS = {"counters": 1, "words": 2}
+# (transport, CTA layout): the counters transport laid out by work where it
+# fits (the default) and on contiguous rank ranges, and flagged words
+SCHED_VARIANTS = {"counters": (1, 0), "counters_ranges": (1, 1), "words": (2, 0)}
 
 
 @pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
-@pytest.mark.parametrize("transport", list(TRANSPORTS))
-def test_schedule_matches_oracle(pkg, orc, case, transport):
+@pytest.mark.parametrize("variant", list(SCHED_VARIANTS))
+def test_schedule_matches_oracle(pkg, orc, case, variant):
     _, kind, seed, p, m, kw, blist = case
+    transport, layout = SCHED_VARIANTS[variant]
     dev = torch.device("cuda:0")
     x = host_inputs(kind, seed, p, m, **kw)
     want = _want(orc, x, kind)
@@ -106,8 +110,11 @@ def test_schedule_matches_oracle(pkg, orc, case, transport):
     for b in blist:
         ys, _ = empty_like_ranks(xs)
         with pkg.Plan(p, m, kind, b) as plan:
-            plan.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[transport])
-            assert plan.info()["sched_transport"] == TRANSPORTS[transport]
+            plan.set(pkg.OPT_SCHED_TRANSPORT, transport)
+            plan.set(pkg.OPT_SCHED_LAYOUT, layout)
+            assert plan.info()["sched_transport"] == transport
+            if layout == 1:
+                assert plan.info()["sched_layout"] == 1
             plan.allreduce_schedule(xs, ys)
             plan.sync()
         _check_all(ys, want)
@@ -382,8 +389,8 @@ def test_invalid_arguments(pkg):
     ("float32", 32, 65541, 4, 7), ("int32", 7, 1000, 4, 3), ("mat2x2u32", 36, 4099, 16, 5),
     ("float32", 1152, 4099, 3, 2), ("int32", 2, 333, 1, 64), ("float32", 1, 17, 2, 3)])
 @pytest.mark.parametrize("layout", ["aligned", "in_place", "four_byte"])
-@pytest.mark.parametrize("transport", list(TRANSPORTS))
-def test_schedule_column_slices(pkg, orc, kind, p, m, b, slices, layout, transport):
+@pytest.mark.parametrize("variant", list(SCHED_VARIANTS))
+def test_schedule_column_slices(pkg, orc, kind, p, m, b, slices, layout, variant):
     """Several CTAs per virtual rank, each running the schedule on its own
     column slice of every block, give the same bits."""
     x = host_inputs(kind, 61, p, m)
@@ -394,11 +401,50 @@ def test_schedule_column_slices(pkg, orc, kind, p, m, b, slices, layout, transpo
     ys, keep_y = (xs, None) if layout == "in_place" else empty_like_ranks(xs, pad_front=pad)
     with pkg.Plan(p, m, kind, b) as plan:
         plan.set(pkg.OPT_SCHED_SLICES, slices)
-        plan.set(pkg.OPT_SCHED_TRANSPORT, TRANSPORTS[transport])
+        plan.set(pkg.OPT_SCHED_TRANSPORT, SCHED_VARIANTS[variant][0])
+        plan.set(pkg.OPT_SCHED_LAYOUT, SCHED_VARIANTS[variant][1])
         assert plan.info()["sched_slices"] == slices
         plan.allreduce_schedule(xs, ys)
         plan.sync()
     _check_all(ys, want)
+
+
+def test_schedule_layout_choice(pkg, orc):
+    """The counters kernels lay ranks out by work (one rank per group: a
+    leaf on one warp beside an inner node on three, each root on a CTA of its
+    own) while one column slice of that fits the GPU at once, and on rank
+    ranges otherwise; forcing the work layout where it does not fit is
+    refused and leaves the plan as it was."""
+    from paper_2109_12626_gb300 import DpdrError
+    for p, want in ((7, 2), (32, 2), (36, 2), (1152, 2), (2, 2), (1, 2), (8190, 1)):
+        with pkg.Plan(p, 1 << 16, "int32", 64) as plan:
+            plan.set(pkg.OPT_SCHED_TRANSPORT, 1)
+            info = plan.info()
+            assert info["sched_layout"] == want, p
+            if want == 2:
+                assert info["sched_ranks_per_cta"] <= 4
+                assert info["sched_ctas"] % info["sched_slices"] == 0
+    with pkg.Plan(32, 1 << 16, "int32", 64) as plan:
+        plan.set(pkg.OPT_SCHED_TRANSPORT, 1)
+        plan.set(pkg.OPT_SCHED_LAYOUT, 1)
+        assert plan.info()["sched_layout"] == 1
+        plan.set(pkg.OPT_SCHED_LAYOUT, 2)
+        assert plan.info()["sched_layout"] == 2
+        plan.set(pkg.OPT_SCHED_RANKS_PER_CTA, 2)  # ranks per CTA: rank ranges
+        assert plan.info()["sched_layout"] == 1
+    kind, p, m = "int32", 8190, 33
+    x = host_inputs(kind, 73, p, m, lo=-1000, hi=1000)
+    xs, _ = to_device(x, kind, torch.device("cuda:0"))
+    ys, _ = empty_like_ranks(xs)
+    with pkg.Plan(p, m, kind, 2) as plan:
+        plan.set(pkg.OPT_SCHED_TRANSPORT, 1)
+        before = plan.info()
+        with pytest.raises(DpdrError):
+            plan.set(pkg.OPT_SCHED_LAYOUT, 2)
+        assert plan.info() == before
+        plan.allreduce_schedule(xs, ys)
+        plan.sync()
+    _check_all(ys, _want(orc, x, kind))
 
 
 def test_schedule_transport_choice(pkg):
@@ -420,6 +466,9 @@ def test_schedule_transport_choice(pkg):
             assert plan.info()["sched_transport"] == 2
     for p in (2048, 4094):
         with pkg.Plan(p, 1, "int32", 0) as plan:
+            # the rule counts ranks per CTA of rank ranges at 128 threads
+            plan.set(pkg.OPT_SCHED_THREADS, 128)
+            plan.set(pkg.OPT_SCHED_LAYOUT, 1)
             rpc = plan.info()["sched_ranks_per_cta"]
             want = 2 if rpc <= 2 else 1
             assert plan.info()["sched_transport"] == want, (p, rpc)
