@@ -709,6 +709,30 @@ def main(argv=None) -> int:
     achieved = algo_bytes / (avg_launch * 1e-3) / 1e9
     peak, peak_kind = measured_peak_gbs()
     units = p * m
+    # small workloads start every step cold: a plain device copy of the same
+    # bytes (p m esize read, as many written), timed the same way after the
+    # same L2 flush, is the floor that method allows
+    copy_ref = None
+    if flush is not None and rank == 0:
+        src_t = torch.empty(p * m * es // 4, dtype=torch.int32, device=dev)
+        dst_t = torch.empty_like(src_t)
+        for _ in range(3):
+            dst_t.copy_(src_t)
+        cts = []
+        for k in range(args.steps):
+            flush.fill_(k + 1)
+            a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a0.record(stream)
+            dst_t.copy_(src_t)
+            a1.record(stream)
+            torch.cuda.synchronize(dev)
+            cts.append(a0.elapsed_time(a1))
+        copy_us = 1000 * sum(cts) / len(cts)
+        copy_ref = {"us": round(copy_us, 2), "kernel_us": round(1000 * avg_launch, 2),
+                    "kernel_over_copy": round(1000 * avg_launch / copy_us, 3),
+                    "what": "torch device copy of p*m*esize bytes, L2 flushed before each, "
+                            "mean of the same number of steps"}
+        del src_t, dst_t
 
     # end to end with host buffers
     e2e = None
@@ -789,6 +813,7 @@ def main(argv=None) -> int:
         "e2e": e2e,
         "gpu_launches": args.steps * launches_per_step,
         "clocks": clocks,
+        "cold_copy_reference": copy_ref,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
