@@ -204,7 +204,14 @@ int dpdr_plan_query(dpdr_plan_t plan, int* parent, int* child0, int* child1,
  *                             whole CTA), DPDR_ERR_INVALID when one column
  *                             slice of it does not fit the GPU at once;
  *                             0 (default) takes 2 where it fits, else 1.
- *                             Set ranks per CTA always take rank ranges */
+ *                             Set ranks per CTA always take rank ranges
+ *   DPDR_OPT_SCHED_COPY       how the counters transport's block passes move
+ *                             16-byte units (same result either way):
+ *                             1 per-lane copies into private shared-memory
+ *                             slots; 2 bulk (TMA) copies of chunks of a few KB
+ *                             through a double-buffered region per rank;
+ *                             0 (default) takes 1 while a column slice of a
+ *                             block holds at most 1024 units, else 2 */
 enum {
     DPDR_OPT_FUSED_MODE = 1,
     DPDR_OPT_WAIT_LIMIT_NS = 2,
@@ -217,7 +224,8 @@ enum {
     DPDR_OPT_HOST_CHUNK_BYTES = 9,
     DPDR_OPT_HOST_PATH = 10,
     DPDR_OPT_SCHED_TRANSPORT = 11,
-    DPDR_OPT_SCHED_LAYOUT = 12
+    DPDR_OPT_SCHED_LAYOUT = 12,
+    DPDR_OPT_SCHED_COPY = 13
 };
 int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
 
@@ -236,7 +244,9 @@ int dpdr_plan_set(dpdr_plan_t plan, int key, int64_t value);
  *        device buffers (8 while those CTAs fit in one wave of resident
  *        CTAs, 2 per SM; else 16; host buffers always take 8)
  *   [17] CTA layout of the schedule kernels: 1 rank ranges, 2 by work
- *        (DPDR_OPT_SCHED_LAYOUT; flagged words always take rank ranges) */
+ *        (DPDR_OPT_SCHED_LAYOUT; flagged words always take rank ranges)
+ *   [18] block passes of the counters transport: 1 per-lane copies, 2 bulk
+ *        copies (DPDR_OPT_SCHED_COPY) */
 int dpdr_plan_info(dpdr_plan_t plan, int64_t* info, int n);
 
 /* Releases the plan's device and host memory.  The caller must first make

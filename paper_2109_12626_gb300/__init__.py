@@ -15,7 +15,7 @@ from ._native import (DPDR_ERR_CUDA, DPDR_ERR_INVALID,  # noqa: F401
                       DPDR_OP_MATMUL, DPDR_OP_SUM, OPT_BLOCKS, OPT_FUSED_MODE,
                       OPT_HOST_CHUNK_BYTES, OPT_HOST_PATH,
                       OPT_SCHED_RANKS_PER_CTA, OPT_SCHED_SLICES,
-                      OPT_SCHED_LAYOUT, OPT_SCHED_THREADS, OPT_SCHED_TRANSPORT,
+                      OPT_SCHED_COPY, OPT_SCHED_LAYOUT, OPT_SCHED_THREADS, OPT_SCHED_TRANSPORT,
                       OPT_SKIP_RANK, OPT_SPLIT_DEPTH, OPT_WAIT_LIMIT_NS, DpdrError,
                       Plan,
                       block_count_rule, blocks, lib, tree)

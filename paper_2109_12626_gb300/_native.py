@@ -19,7 +19,7 @@ DPDR_OP_SUM, DPDR_OP_MATMUL = 0, 1
 (OPT_FUSED_MODE, OPT_WAIT_LIMIT_NS, OPT_SKIP_RANK, OPT_SCHED_THREADS,
  OPT_SCHED_RANKS_PER_CTA, OPT_BLOCKS, OPT_SPLIT_DEPTH, OPT_SCHED_SLICES,
  OPT_HOST_CHUNK_BYTES, OPT_HOST_PATH, OPT_SCHED_TRANSPORT,
- OPT_SCHED_LAYOUT) = range(1, 13)
+ OPT_SCHED_LAYOUT, OPT_SCHED_COPY) = range(1, 14)
 
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libdpdr.so")
 
@@ -145,7 +145,7 @@ INFO_KEYS = ("p", "m", "b", "max_depth", "auto_mode", "sched_ctas",
              "sched_ranks_per_cta", "scratch_bytes", "vector_path",
              "split_depth", "split_subtrees", "split_group", "sched_slices",
              "topology", "host_path", "sched_transport", "tree_width",
-             "sched_layout")
+             "sched_layout", "sched_copy")
 
 
 class Plan:

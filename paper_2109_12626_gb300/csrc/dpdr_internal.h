@@ -87,6 +87,7 @@ struct Plan {
     int split_depth = -1;      // cut depth of the split layout, -1 = auto
     int sched_transport = 0;   // schedule kernel: 0 auto, 1 counters, 2 flagged words
     int sched_layout = 0;      // counters kernels' CTA layout: 0 auto, 1 rank ranges, 2 by work
+    int sched_copy = 0;        // counters kernels' block passes: 0 auto, 1 per-lane, 2 bulk
     int64_t host_chunk = int64_t(1) << 30;  // bytes of rank data per host-pipeline chunk
     int host_path = 0;         // dpdr_allreduce_host: 0 auto, 1 copy pipeline, 2 direct
     int last_host_path = 0;    // path the last dpdr_allreduce_host took (1 or 2)
@@ -163,6 +164,7 @@ struct Plan {
     int sched_threads_used = 128;  // threads per CTA of the kernel that runs
     int sched_slices_used = 1, sched_chunks = 1;
     int sched_layout_used = 1;     // 1 rank ranges, 2 by work
+    int sched_copy_used = 2;       // 1 per-lane copies, 2 bulk copies
     int sched_slot_bytes = 192;    // counters kernels: shared memory per thread
 };
 

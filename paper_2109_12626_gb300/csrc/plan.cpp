@@ -465,6 +465,10 @@ extern "C" int dpdr_plan_set(dpdr_plan_t h, int key, int64_t v)
         }
         return rc;
     }
+    case DPDR_OPT_SCHED_COPY:
+        if (v < 0 || v > 2) return fail(DPDR_ERR_INVALID, "schedule copy: 0, 1 or 2");
+        P->sched_copy = int(v);
+        return schedule_configure(P);
     case DPDR_OPT_SCHED_SLICES:
         if (v < 0 || v > kMaxSlices) return fail(DPDR_ERR_INVALID, "slices: 0..1024");
         P->sched_slices = int(v);
@@ -524,7 +528,7 @@ extern "C" int dpdr_plan_info(dpdr_plan_t h, int64_t* info, int n)
                          P->last_vector_path, P->split_s, P->split_nseg, P->split_group,
                          P->sched_slices_used, P->topo, P->last_host_path,
                          schedule_transport(P), P->tree[fused_tree_index(P)].width,
-                         P->sched_layout_used};
+                         P->sched_layout_used, P->sched_copy_used};
     const int k = int(sizeof v / sizeof v[0]);
     for (int i = 0; i < n; i++) info[i] = i < k ? v[i] : 0;
     return DPDR_OK;

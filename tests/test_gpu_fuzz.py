@@ -47,6 +47,7 @@ def draw(k: int) -> dict:
     # the schedule kernels' CTA layout: automatic (by work where it fits) or
     # rank ranges, drawn last so the draws above stay as they were
     c["sched_layout"] = 1 if rng.random() < 0.3 else 0
+    c["sched_copy"] = int(rng.integers(0, 3))  # drawn after the layout, as above
     return c
 
 
@@ -96,6 +97,7 @@ def test_random_configuration(pkg, orc, k):
             else:
                 plan.set(pkg.OPT_SCHED_TRANSPORT, c["transport"])
                 plan.set(pkg.OPT_SCHED_LAYOUT, c["sched_layout"])
+                plan.set(pkg.OPT_SCHED_COPY, c["sched_copy"])
                 if c["slices"]:
                     plan.set(pkg.OPT_SCHED_SLICES, c["slices"])
                 if c["rpc"]:
@@ -130,6 +132,7 @@ def draw_large(k: int) -> dict:
              mode=int(rng.integers(0, 6)), transport=int(rng.choice([0, 1, 1, 2])),
              slices=int(rng.integers(1, 33)) if rng.random() < 0.5 else 0)
     c["sched_layout"] = 1 if rng.random() < 0.3 else 0  # drawn last, as above
+    c["sched_copy"] = int(rng.integers(0, 3))
     return c
 
 
@@ -167,6 +170,7 @@ def test_random_large_configuration(pkg, orc, k):
             else:
                 plan.set(pkg.OPT_SCHED_TRANSPORT, c["transport"])
                 plan.set(pkg.OPT_SCHED_LAYOUT, c["sched_layout"])
+                plan.set(pkg.OPT_SCHED_COPY, c["sched_copy"])
                 if c["slices"]:
                     plan.set(pkg.OPT_SCHED_SLICES, c["slices"])
                 plan.allreduce_schedule(xs, list(yt.unbind(0)))

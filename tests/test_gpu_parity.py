@@ -93,16 +93,20 @@ def test_fused_matches_oracle(pkg, orc, case, mode):
 
 
 TRANSPORTS = {"counters": 1, "words": 2}
-# (transport, CTA layout): the counters transport laid out by work where it
-# fits (the default) and on contiguous rank ranges, and flagged words
-SCHED_VARIANTS = {"counters": (1, 0), "counters_ranges": (1, 1), "words": (2, 0)}
+# (transport, CTA layout, block-pass copies): the counters transport laid out
+# by work where it fits (the default) and on contiguous rank ranges, its block
+# passes by per-lane copies (the automatic choice at these sizes) and by bulk
+# copies, and flagged words
+SCHED_VARIANTS = {"counters": (1, 0, 0), "counters_bulk": (1, 0, 2),
+                  "counters_ranges_lane": (1, 1, 1), "counters_ranges_bulk": (1, 1, 2),
+                  "words": (2, 0, 0)}
 
 
 @pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
 @pytest.mark.parametrize("variant", list(SCHED_VARIANTS))
 def test_schedule_matches_oracle(pkg, orc, case, variant):
     _, kind, seed, p, m, kw, blist = case
-    transport, layout = SCHED_VARIANTS[variant]
+    transport, layout, copy = SCHED_VARIANTS[variant]
     dev = torch.device("cuda:0")
     x = host_inputs(kind, seed, p, m, **kw)
     want = _want(orc, x, kind)
@@ -112,9 +116,12 @@ def test_schedule_matches_oracle(pkg, orc, case, variant):
         with pkg.Plan(p, m, kind, b) as plan:
             plan.set(pkg.OPT_SCHED_TRANSPORT, transport)
             plan.set(pkg.OPT_SCHED_LAYOUT, layout)
+            plan.set(pkg.OPT_SCHED_COPY, copy)
             assert plan.info()["sched_transport"] == transport
             if layout == 1:
                 assert plan.info()["sched_layout"] == 1
+            if copy:
+                assert plan.info()["sched_copy"] == copy
             plan.allreduce_schedule(xs, ys)
             plan.sync()
         _check_all(ys, want)
@@ -403,6 +410,7 @@ def test_schedule_column_slices(pkg, orc, kind, p, m, b, slices, layout, variant
         plan.set(pkg.OPT_SCHED_SLICES, slices)
         plan.set(pkg.OPT_SCHED_TRANSPORT, SCHED_VARIANTS[variant][0])
         plan.set(pkg.OPT_SCHED_LAYOUT, SCHED_VARIANTS[variant][1])
+        plan.set(pkg.OPT_SCHED_COPY, SCHED_VARIANTS[variant][2])
         assert plan.info()["sched_slices"] == slices
         plan.allreduce_schedule(xs, ys)
         plan.sync()
@@ -445,6 +453,22 @@ def test_schedule_layout_choice(pkg, orc):
         plan.allreduce_schedule(xs, ys)
         plan.sync()
     _check_all(ys, _want(orc, x, kind))
+
+
+def test_schedule_copy_choice(pkg):
+    """Block passes by per-lane copies while a column slice of a block holds
+    at most 1024 16-byte units, by bulk copies beyond; the option forces
+    either, and other values are refused."""
+    from paper_2109_12626_gb300 import DpdrError
+    for p, m, b, want in ((32, 1 << 23, 64, 1), (32, 1 << 23, 16, 2), (1152, 1 << 18, 18, 2),
+                          (1152, 1 << 18, 72, 1), (32, 1 << 27, 1024, 1), (32, 1 << 27, 256, 2)):
+        with pkg.Plan(p, m, "float32", b) as plan:
+            plan.set(pkg.OPT_SCHED_TRANSPORT, 1)
+            assert plan.info()["sched_copy"] == want, (p, m, b)
+            plan.set(pkg.OPT_SCHED_COPY, 3 - want)
+            assert plan.info()["sched_copy"] == 3 - want
+            with pytest.raises(DpdrError):
+                plan.set(pkg.OPT_SCHED_COPY, 3)
 
 
 def test_schedule_transport_choice(pkg):

@@ -35,7 +35,8 @@ CASES = [("float32", 1, 33, 1), ("float32", 2, 1001, 3), ("int32", 3, 17, 17),
 
 @pytest.mark.parametrize("kind,p,m,b", CASES)
 @pytest.mark.parametrize("layout", ["auto", "slices", "groups"])
-def test_reduce_bcast_parity(pkg, orc, kind, p, m, b, layout):
+@pytest.mark.parametrize("copy", [0, 2], ids=["copy_auto", "copy_bulk"])
+def test_reduce_bcast_parity(pkg, orc, kind, p, m, b, layout, copy):
     x = host_inputs(kind, 91, p, m)
     want = expect_bits(orc.tree_fold(x, _dt(orc, kind), orc.SINGLE))
     dev = torch.device("cuda:0")
@@ -46,6 +47,7 @@ def test_reduce_bcast_parity(pkg, orc, kind, p, m, b, layout):
             plan.set(pkg.OPT_SCHED_SLICES, 3)
         if layout == "groups":
             plan.set(pkg.OPT_SCHED_RANKS_PER_CTA, min(p, 3))
+        plan.set(pkg.OPT_SCHED_COPY, copy)
         plan.allreduce_reduce_bcast(xs, ys)
         plan.sync()
     for i, y in enumerate(ys):
