@@ -237,15 +237,18 @@ def profiled_traffic(kernel: str, wname: str, units: int,
     path = os.path.join(ROOT, "profiles", "traffic.json")  # ncu figures, not code
     try:
         with open(path) as f:
-            rec = json.load(f)[kernel][wname]
+            recs = json.load(f)[kernel][wname]
     except (OSError, KeyError, ValueError):
         return None
-    if rec.get("source_hash") != kernel_source_hash(kernel):
-        return None
-    want = rec.get("block_elems")
-    if want is not None and (block is None or abs(block - want) > 0.05 * want):
-        return None
-    return float(rec["bytes_per_unit"]) * units
+    # one record, or (schedule kernel) a list of records for several block sizes
+    for rec in recs if isinstance(recs, list) else [recs]:
+        if rec.get("source_hash") != kernel_source_hash(kernel):
+            continue
+        want = rec.get("block_elems")
+        if want is not None and (block is None or abs(block - want) > 0.05 * want):
+            continue
+        return float(rec["bytes_per_unit"]) * units
+    return None
 
 
 # --------------------------------------------------------- CPU oracle
