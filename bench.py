@@ -474,6 +474,8 @@ def run_sweep(args, w) -> int:
             b0 = -(-m // args.block_size) if args.block_size else 0
             with pkg.Plan(p, m, kind, b0, topology=args.topology) as plan:
                 set_schedule_options(pkg, plan, args)
+                if args.split_depth is not None:
+                    plan.set(pkg.OPT_SPLIT_DEPTH, args.split_depth)
                 if args.mode:
                     plan.set(pkg.OPT_FUSED_MODE, args.mode)
                 bd = plan.bind(xs, ys)
