@@ -265,10 +265,12 @@ int dpdr_allreduce(dpdr_plan_t plan, const void* const* x, void* const* y,
 
 /* Schedule-faithful kernel: runs Algorithm 1 for every virtual rank, rounds
  * j = 0..b+d_i, each round's exchanges with child_0, child_1 and the parent
- * or dual, as one cooperative persistent launch in which CTAs own ranks and
- * exchange pipeline blocks through device memory, published either by
- * release/acquire counters or as epoch-flagged words
- * (DPDR_OPT_SCHED_TRANSPORT).  Same result as dpdr_allreduce.  Two calls
+ * or dual, as one cooperative persistent launch in which groups of warps
+ * serve ranks (DPDR_OPT_SCHED_LAYOUT) and exchange pipeline blocks through
+ * device memory, published either by release/acquire counters or as
+ * epoch-flagged words (DPDR_OPT_SCHED_TRANSPORT); with counters, blocks
+ * move between device memory and shared memory by bulk (TMA) or per-lane
+ * copies (DPDR_OPT_SCHED_COPY).  Same result as dpdr_allreduce.  Two calls
  * on one plan that overlap on the GPU (two streams) race on its scratch.  Every wait is bounded
  * (DPDR_OPT_WAIT_LIMIT_NS); an expired wait ends the kernel early and is
  * reported as DPDR_ERR_TIMEOUT by dpdr_plan_sync.  Returns
