@@ -68,7 +68,8 @@ static int64_t stream_target(const Plan* P) { return int64_t(P->num_sms) * 1024;
 //    needs to fill the GPU (p = 36, 2x2 matrices, m = 2^16: 13 us against the
 //    tile's 15 us; 32768 int32 units: p = 64, 14.6 against 17.2 us, p = 127,
 //    28.4 against 32.5), and the shared-memory tile below that (8192 units:
-//    p = 64, 7.8 against 11.3 us; p = 127, 9.5 against 25.1).
+//    p = 64, 7.8 against 11.3 us; p = 127, 9.5 against 25.1) unless the
+//    trees are shallow (p <= 16: column streaming at every size).
 constexpr int64_t kTileMaxBytes = int64_t(40) << 20;
 constexpr int kSplitMinRanks = 128;
 constexpr int64_t kSplitWork = int64_t(1) << 17;
@@ -80,6 +81,8 @@ constexpr int64_t kTreeMinBytesLargeP = int64_t(20) << 20;
 // against 6.2/8.2); above it the hierarchical tile leads cold (p = 576,
 // m = 8192: 14.5 against 17.0 us).
 constexpr int64_t kTileOverTreeUnits = 1024;
+// Up to this many ranks column streaming takes even the fewest columns.
+constexpr int kStreamMaxShallowRanks = 16;
 
 // Resident CTAs of the shared-memory tile on the GPU: up to 4 per SM (256
 // threads of 64 registers), fewer when its rows do not fit the 228 KB of
@@ -146,6 +149,11 @@ int fused_auto_mode(const Plan* P)
     if (tile_preferred(P)) return 2;
     if (P->p >= kSplitMinRanks && units >= 4096 && P->split_ready) return 3;
     if (units >= stream_target(P) / 5) return 1;
+    // shallow trees: a column's walk is a batch or two of loads, and column
+    // streaming beats staging rows through the tile (cold, p = 7, m = 1000
+    // int32: 6.8 against 8.9 us; at p <= 16 it is never slower, from p = 32
+    // the tile leads)
+    if (P->p <= kStreamMaxShallowRanks) return 1;
     if (tile_lg_wu(P) >= 0) return 2;
     return P->split_ready ? 3 : 1;
 }

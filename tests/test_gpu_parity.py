@@ -199,7 +199,7 @@ def test_guard_words_untouched(pkg, orc, run):
 
 AUTO = [  # p, m, kind, layout the automatic choice takes on a 152-SM GPU
           # (1 stream, 2 tile, 3 split, 5 hierarchical tile)
-    (32, 1 << 27, "float32", 1), (36, 65536, "mat2x2u32", 1), (7, 1000, "int32", 2),
+    (32, 1 << 27, "float32", 1), (36, 65536, "mat2x2u32", 1),
     (1152, 4096, "int32", 2), (1152, 8192, "int32", 5), (1152, 32768, "int32", 5),
     (288, 4096, "int32", 2), (288, 4100, "int32", 5), (768, 4096, "int32", 2),
     (1152, 32772, "int32", 3), (128, 16384, "float32", 5), (192, 32768, "int32", 2),
@@ -212,6 +212,8 @@ AUTO = [  # p, m, kind, layout the automatic choice takes on a 152-SM GPU
     # below p = 128: column streaming from a fifth of the columns that fill
     # the GPU (31129 units on 152 SMs), the shared-memory tile below
     (64, 131072, "int32", 1), (64, 65536, "int32", 2),
+    # shallow trees (p <= 16): column streaming at every size
+    (7, 1000, "int32", 1), (16, 16, "int32", 1), (2, 3, "float32", 1), (32, 1000, "int32", 2),
     # from p = 2048 the split layout where the wide hierarchical tile's second
     # wave would be less than 60 % full
     (4094, 24576, "int32", 3), (4094, 32768, "int32", 5), (2304, 20480, "int32", 3),
