@@ -16,8 +16,9 @@
 // has published, down[i] = number of final blocks it holds.  A send is a
 // release store of the counter after the block is written; a receive is an
 // acquire load of the partner's counter followed by reading the partner's
-// block straight from the partner's buffer (L2-coherent loads), fused with
-// the (.) -- the temporary t of Algorithm 1 never materialises.  Where a
+// block straight from the partner's buffer (bulk or per-lane copies into
+// shared memory, served by L2), fused with the (.) -- the temporary t of
+// Algorithm 1 never materialises in device memory.  Where a
 // partial lives: a leaf's partial block j is x_i[j] itself, an inner node's
 // is y_i[j], a root's is one of two exchange slots per root (the dual reads
 // it while the root overwrites y_r[j] with the final block).  A child

@@ -10,7 +10,7 @@ namespace dpdr {
 namespace sched {
 
 constexpr int kMaxThreads = 256;
-constexpr int kMaxGroups = 4;  // rank groups per CTA (named barriers 1..4)
+constexpr int kMaxGroups = 4;  // rank groups per CTA
 
 // Rank groups of a CTA that owns R virtual ranks: min(R, warps, kMaxGroups)
 // groups of whole warps, all of one size, each running its own ranks.
