@@ -73,7 +73,9 @@ def _sampled_check(orc, w, m, xs, ys, cols):
 
 
 @pytest.mark.parametrize("name,kernels", [
-    ("p32_m134217728_f32", ("fused", "schedule")),
+    # at the workload's b = 1024 the schedule kernel's column slices are short
+    # (per-lane copies); at the plan's default b they are long (bulk copies)
+    ("p32_m134217728_f32", ("fused", "schedule", "schedule_default_b")),
     ("p1152_m4194304_f32", ("fused", "schedule")),
     ("p36_m65536_mat2x2u32", ("fused", "schedule")),
     ("p36_m65536_mat2x2f32", ("fused", "schedule")),
@@ -85,10 +87,9 @@ def test_full_size_workloads(pkg, orc, name, kernels):
     dev = torch.device("cuda:0")
     xs = _device_inputs(w, m, dev)
     ys = [torch.empty_like(x) for x in xs]
-    with pkg.Plan(p, m, w["kind"], w.get("b") or 0) as plan:
-        b = plan.query()["b"]
-        cols = _columns(m, b)
-        for k in kernels:
+    for k in kernels:
+        with pkg.Plan(p, m, w["kind"], 0 if k == "schedule_default_b" else w.get("b") or 0) as plan:
+            cols = _columns(m, plan.query()["b"])
             for y in ys:
                 y.fill_(-1)
             (plan.allreduce if k == "fused" else plan.allreduce_schedule)(xs, ys)
