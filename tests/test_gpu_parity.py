@@ -457,6 +457,36 @@ def test_schedule_layout_choice(pkg, orc):
     _check_all(ys, _want(orc, x, kind))
 
 
+@pytest.mark.parametrize("p", [2400, 2432, 2600])
+def test_schedule_layout_at_its_limit(pkg, orc, p):
+    """On both sides of the largest p whose work layout fits one slice of
+    resident CTAs (128-thread CTAs, 8 per SM: a leaf and an inner node per
+    CTA, a CTA per root, spare leaves four to a CTA), the automatic layout
+    gives the same bits as the oracle; the work layout, where taken, has the
+    CTAs per slice that its rule counts, and it is not taken where those
+    cannot all reside."""
+    kind, m = "int32", 37
+    x = host_inputs(kind, 81, p, m, lo=-1000, hi=1000)
+    xs, _ = to_device(x, kind, torch.device("cuda:0"))
+    ys, _ = empty_like_ranks(xs)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    with pkg.Plan(p, m, kind, 3) as plan:
+        plan.set(pkg.OPT_SCHED_TRANSPORT, 1)
+        info = plan.info()
+        par = plan.query()["parent"]
+        c0 = plan.query()["child0"]
+        leaves = sum(1 for i in range(p) if par[i] >= 0 and c0[i] < 0)
+        inner = sum(1 for i in range(p) if par[i] >= 0 and c0[i] >= 0)
+        ctas = 2 + inner + -(-(leaves - min(leaves, inner)) // 4)
+        if ctas > 8 * sms:  # more than the 64-register budget lets reside
+            assert info["sched_layout"] == 1, (p, ctas)
+        if info["sched_layout"] == 2:
+            assert info["sched_ctas"] == ctas * info["sched_slices"], (p, ctas)
+        plan.allreduce_schedule(xs, ys)
+        plan.sync()
+    _check_all(ys, _want(orc, x, kind))
+
+
 def test_schedule_copy_choice(pkg):
     """Block passes by per-lane copies while a column slice of a block holds
     at most 1024 16-byte units, by bulk copies beyond; the option forces
